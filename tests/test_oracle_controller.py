@@ -1,0 +1,214 @@
+"""Pins for the oracle's controller (Algorithm 1, Sec. 3.3) and step loop.
+
+The golden cases in tests/golden/controller_cases.json were worked by hand
+from Algorithm 1; the invariants below follow from it (proofs in the
+docstrings) and do not re-run the oracle's own formula.
+"""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import acid_synth as S
+import oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "controller_cases.json")
+
+
+def _run(signals, warmup, tl, th, delta):
+    ctl = O.AcidController(tl, th, delta)
+    comp, taus, sig = [], [], []
+    for i, s in enumerate(signals):
+        if i < warmup:
+            comp.append(True)
+            taus.append(None)
+            sig.append(None)
+            continue
+        skip, tau, sg, _ = ctl.step(s)
+        comp.append(not skip)
+        taus.append(tau)
+        sig.append(sg)
+    return comp, taus, sig
+
+
+@pytest.mark.parametrize("case", json.load(open(GOLDEN))["cases"], ids=lambda c: c["name"])
+def test_golden_cases(case):
+    comp, taus, sig = _run(case["signals"], case["warmup"], case["tau_low"], case["tau_high"],
+                           case["delta"])
+    assert comp == case["computed"]
+    for a, b in zip(taus, case["tau"]):
+        assert (a is None and b is None) or a == pytest.approx(b, abs=1e-12)
+    for a, b in zip(sig, case["sigma"]):
+        assert (a is None and b is None) or a == pytest.approx(b, abs=1e-12)
+
+
+def _fixed_tau(signals, warmup, tau):
+    """Fixed-threshold caching skeleton (Sec. 2, 'The Fixed Threshold...'):
+    accumulate, reuse while the sum stays within tau, else run and reset."""
+    acc = 0.0
+    out = []
+    for i, s in enumerate(signals):
+        if i < warmup:
+            out.append(True)
+            continue
+        acc += s
+        if acc <= tau:
+            out.append(False)
+        else:
+            out.append(True)
+            acc = 0.0
+    return out
+
+
+def _random_signals(rng, n):
+    # piecewise-smooth non-negative sequences with occasional jumps
+    base = rng.uniform(0.0, 0.1)
+    s = []
+    for _ in range(n):
+        if rng.uniform() < 0.25:
+            base = rng.uniform(0.0, 0.15)
+        s.append(max(0.0, base + rng.normal(0, 0.01)))
+    return s
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_equal_thresholds_reduce_to_fixed_tau(seed):
+    """tau_low == tau_high: the threshold no longer depends on the signal's
+    rate of change, so ACID is the fixed-threshold method (Sec. 3.3)."""
+    rng = np.random.default_rng(seed)
+    s = _random_signals(rng, 50)
+    tau = rng.uniform(0.02, 0.3)
+    delta = rng.uniform(-0.05, 0.05)
+    w = int(rng.integers(0, 3))
+    assert O.controller_decisions(s, w, tau, tau, delta) == _fixed_tau(s, w, tau)
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_negative_delta_is_fixed_low(seed):
+    """delta < 0 makes |s_t - s_prev| <= delta impossible: always tau_low."""
+    rng = np.random.default_rng(100 + seed)
+    s = _random_signals(rng, 50)
+    tl, th = sorted(rng.uniform(0.02, 0.4, size=2))
+    assert O.controller_decisions(s, 1, tl, th, -1.0) == _fixed_tau(s, 1, tl)
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_compute_count_between_fixed_thresholds(seed):
+    """For non-negative signals the active threshold tau_t lies in
+    [tau_low, tau_high] and depends on the signals only (s_prev is updated on
+    every non-warmup step).  Greedy accumulate-and-reset with pointwise larger
+    thresholds never computes earlier: if the k-th compute under the larger
+    schedule is at e', the smaller schedule has accumulated at least the same
+    segment sum by e' and so has computed k times by then.  Hence
+    #computed(fixed tau_high) <= #computed(ACID) <= #computed(fixed tau_low)."""
+    rng = np.random.default_rng(200 + seed)
+    s = _random_signals(rng, 60)
+    tl, th = sorted(rng.uniform(0.01, 0.4, size=2))
+    delta = rng.uniform(0.0, 0.05)
+    a = sum(O.controller_decisions(s, 1, tl, th, delta))
+    lo = sum(_fixed_tau(s, 1, tl))
+    hi = sum(_fixed_tau(s, 1, th))
+    assert hi <= a <= lo
+
+
+def test_zero_signal_skips_everything():
+    d = O.controller_decisions([0.0] * 20, 2, 0.05, 0.2, 0.01)
+    assert d == [True, True] + [False] * 18
+
+
+def test_infinite_signal_forces_compute():
+    d = O.controller_decisions([0.0, math.inf, 0.0, math.inf], 1, 1e9, 1e9, 1.0)
+    assert d == [True, True, False, True]
+
+
+def test_forced_decision_overrides_and_updates_state():
+    ctl = O.AcidController(0.1, 0.1, 0.0)
+    skip, _, sg, _ = ctl.step(0.5, forced=False)  # would compute; forced reuse keeps Sigma
+    assert skip and sg == 0.5 and ctl.sigma == 0.5
+    skip, _, sg, _ = ctl.step(0.0, forced=True)  # would skip? 0.5 > 0.1 computes anyway
+    assert not skip and ctl.sigma == 0.0
+    skip, _, _, _ = ctl.step(0.01, forced=True)
+    assert not skip and ctl.sigma == 0.0
+
+
+# ---------------------------------------------------------------------------
+# Loop-level pins on the toy workload
+# ---------------------------------------------------------------------------
+
+@pytest.fixture(scope="module")
+def toy():
+    cfg = S.get_config("toy", steps=6)
+    return cfg, S.model_weights(cfg, 0), S.latent(cfg, 0)
+
+
+def _plain_sampler(cfg, w, lat, n):
+    """No caching: every step evaluates the denoiser (Eq. 2 as Euler)."""
+    sig = O.sigmas(n)
+    x = lat.astype(np.float64)
+    for i in range(n):
+        v = O.denoiser(cfg, w, x, 1000.0 * sig[i], None)
+        x = x + (sig[i + 1] - sig[i]) * v
+    return x
+
+
+def test_loop_negative_threshold_is_uncached(toy):
+    cfg, w, lat = toy
+    r = O.denoise_loop(cfg, w, lat, None, tau_low=-1.0, tau_high=-1.0)
+    assert all(r.computed)
+    np.testing.assert_allclose(r.latent, _plain_sampler(cfg, w, lat, cfg.steps), rtol=0, atol=1e-12)
+
+
+def test_loop_huge_threshold_reuses_first_residual(toy):
+    """With every non-warmup step skipped, TeaCache output is the final layer
+    applied to H_in(x_t) + R_0, where R_0 is the block-stack residual of the
+    first step."""
+    cfg, w, lat = toy
+    r = O.denoise_loop(cfg, w, lat, None, tau_low=1e9, tau_high=1e9)
+    assert r.computed == [True] + [False] * (cfg.steps - 1)
+    sig = O.sigmas(cfg.steps)
+    x = lat.astype(np.float64)
+    si = O.step_inputs(cfg, w, x, 1000.0 * sig[0])
+    R0 = O.block_stack(cfg, w, si.h_in, si.mods, None) - si.h_in
+    for i in range(cfg.steps):
+        si = O.step_inputs(cfg, w, x, 1000.0 * sig[i])
+        v = O.final_layer(cfg, w, si.h_in + R0, si.final_mod)
+        x = x + (sig[i + 1] - sig[i]) * v
+    np.testing.assert_allclose(r.latent, x, rtol=0, atol=1e-12)
+
+
+def test_loop_signals_are_consecutive_temni_drifts(toy):
+    cfg, w, lat = toy
+    r = O.denoise_loop(cfg, w, lat, None)
+    # recompute the TEMNI sequence along the oracle's own trajectory via forced replay
+    forced = [rec.computed for rec in r.records]
+    r2 = O.denoise_loop(cfg, w, lat, None, forced=[None] + forced[1:])
+    assert [x.computed for x in r2.records] == forced
+    np.testing.assert_allclose(r2.latent, r.latent, rtol=0, atol=0)
+    assert all(rec.signal > 0 for rec in r.records[1:])
+
+
+def test_easycache_affine_model_is_exact():
+    """EasyCache (Sec. 2): if the model's output is its input plus a constant
+    offset, k = 1 and the reuse x_t + (v_c - x_c) is exact, so any decision
+    sequence yields the uncached trajectory."""
+    rng = np.random.default_rng(0)
+    c = rng.normal(size=(3, 4))
+    x_c = rng.normal(size=(3, 4))
+    x_prev = x_c - 0.1 * rng.normal(size=(3, 4))
+    k = O.easycache_rate(x_c, x_prev, x_c + c, x_prev + c)
+    assert k == pytest.approx(1.0, abs=1e-15)
+    x_t = x_c + rng.normal(size=(3, 4))
+    np.testing.assert_allclose(O.easycache_reuse(x_t, x_c, x_c + c), x_t + c, atol=1e-15)
+    s = O.easycache_signal(2.0, x_t, x_c, x_c + c)
+    assert s == pytest.approx(2.0 * np.abs(x_t - x_c).mean() / np.abs(x_c + c).mean())
+
+
+def test_easycache_loop_runs_and_warms_up_two_steps():
+    cfg = S.get_config("toy", steps=6, method="easycache", tau_low=0.02, tau_high=0.04)
+    w = S.model_weights(cfg, 1)
+    r = O.denoise_loop(cfg, w, S.latent(cfg, 1), None)
+    assert r.computed[:2] == [True, True]
+    assert all(np.isfinite(rec.signal) for rec in r.records[2:])
