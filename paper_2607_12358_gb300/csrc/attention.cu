@@ -1,0 +1,376 @@
+// Attention over the full spatio-temporal token sequence (self, joint and
+// cross attention of the DiT blocks).  RoPE is applied to q and k once per
+// token by the QKV projection's epilogue, so this kernel reads pre-rotated
+// operands.
+//
+// bf16 path: a flash-attention kernel on tcgen05 tensor cores.  One CTA owns
+// 128 query rows of one head:
+//   warp 0      TMA producer: Q once, then K_j / V_j tiles of 128 keys into a
+//               2-deep ring (128-byte swizzle);
+//   warp 1      MMA issuer: S_j = Q K_j^T into one of two TMEM S buffers,
+//               then O += P_{j-1} V_{j-1} into the TMEM O accumulator, so the
+//               tensor core computes S_{j+1} while softmax works on S_j;
+//   warps 4-7   softmax: one thread per query row reads its S row from TMEM,
+//               keeps the running max and sum, writes P (bf16) to shared
+//               memory in the swizzled K-major layout the MMA reads, and
+//               rescales O in TMEM only when the running max grows by more
+//               than 2^8 (the final division by the sum makes the result
+//               independent of when rescaling happens).
+// fp32 path: one warp per query row, exact expf, for the fp32 mode.
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace acid {
+
+acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
+
+namespace {
+
+constexpr int kBQ = 128;   // query rows per CTA
+constexpr int kBKV = 128;  // keys per tile
+constexpr int kAttnThreads = 256;
+constexpr float kRescaleLog2 = 8.0f;
+
+struct AttnDev {
+  int64_t nq, nk;
+  int q_col, k_col, v_col;
+  void* out;
+  int64_t ldo;
+  int o_col;
+  float scale_log2;  // log2(e) / sqrt(head_dim)
+};
+
+template <int D>
+struct AttnCfg {
+  static constexpr int CH = D / 64;                 // 64-column chunks per row
+  static constexpr int CHUNK_BYTES = 128 * 128;     // 128 rows x 128 bytes
+  static constexpr int Q_BYTES = CH * CHUNK_BYTES;  // also K / V tile bytes
+  static constexpr int P_BYTES = 2 * CHUNK_BYTES;   // 128 x 128 bf16
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + 2 * Q_BYTES;
+  static constexpr int OFF_P = OFF_V + 2 * Q_BYTES;
+  static constexpr int OFF_BAR = OFF_P + P_BYTES;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  static constexpr uint32_t TMEM_COLS = 512;  // S0 [0,128), S1 [128,256), O [256, 256+D)
+  static constexpr uint32_t O_COL = 256;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, AttnDev a) {
+  using C = AttnCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint8_t* sK = smem + C::OFF_K;
+  uint8_t* sV = smem + C::OFF_V;
+  uint8_t* sP = smem + C::OFF_P;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint64_t* q_full = bars + 0;
+  uint64_t* k_full = bars + 1;   // [2]
+  uint64_t* k_empty = bars + 3;  // [2]
+  uint64_t* v_full = bars + 5;   // [2]
+  uint64_t* v_empty = bars + 7;  // [2]
+  uint64_t* s_full = bars + 9;   // [2]
+  uint64_t* s_free = bars + 11;  // [2]
+  uint64_t* p_full = bars + 13;
+  uint64_t* pv_done = bars + 14;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x, h = blockIdx.y;
+  const int nkv = (int)((a.nk + kBKV - 1) / kBKV);
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&v_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], 128);
+    }
+    mbar_init(p_full, 128);
+    mbar_init(pv_done, 1);
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------------------------------- TMA producer
+      mbar_expect_tx(q_full, C::Q_BYTES);
+      for (int c = 0; c < C::CH; ++c)
+        tma_load_2d(sQ + c * C::CHUNK_BYTES, &tmQ, q_full, a.q_col + h * D + c * 64, qt * kBQ);
+      for (int j = 0; j < nkv; ++j) {
+        const int st = j & 1, round = j >> 1;
+        if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) break;
+        mbar_expect_tx(&k_full[st], C::Q_BYTES);
+        for (int c = 0; c < C::CH; ++c)
+          tma_load_2d(sK + st * C::Q_BYTES + c * C::CHUNK_BYTES, &tmK, &k_full[st], a.k_col + h * D + c * 64,
+                      j * kBKV);
+        if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) break;
+        mbar_expect_tx(&v_full[st], C::Q_BYTES);
+        for (int c = 0; c < C::CH; ++c)
+          tma_load_2d(sV + st * C::Q_BYTES + c * C::CHUNK_BYTES, &tmV, &v_full[st], a.v_col + h * D + c * 64,
+                      j * kBKV);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---------------------------------------- MMA issuer
+      constexpr uint32_t idesc_s = idesc_bf16_f32(128, kBKV, false, false);
+      constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
+      bool ok = mbar_wait(q_full, 0);
+      const uint32_t q0 = smem_u32(sQ), p0 = smem_u32(sP);
+      for (int j = 0; ok && j <= nkv; ++j) {
+        if (j < nkv) {
+          const int st = j & 1;
+          if (!mbar_wait(&k_full[st], (j >> 1) & 1)) { ok = false; break; }
+          if (j >= 2 && !mbar_wait(&s_free[st], ((j >> 1) - 1) & 1)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t k0 = smem_u32(sK + st * C::Q_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
+            mma_bf16_ss(tmem + st * kBKV, smem_desc_sw128(q0 + off, 16, 1024), smem_desc_sw128(k0 + off, 16, 1024),
+                        idesc_s, kk != 0);
+          }
+          mma_commit(&k_empty[st]);
+          mma_commit(&s_full[st]);
+        }
+        if (j >= 1) {
+          const int jp = j - 1, st = jp & 1;
+          if (!mbar_wait(p_full, jp & 1)) { ok = false; break; }
+          if (!mbar_wait(&v_full[st], (jp >> 1) & 1)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t v0 = smem_u32(sV + st * C::Q_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < kBKV / 16; ++kk) {
+            const uint32_t poff = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
+            // V is MN-major: 16 key rows of 128 bytes per step; 64-column chunks 16 KB apart
+            mma_bf16_ss(tmem + C::O_COL, smem_desc_sw128(p0 + poff, 16, 1024),
+                        smem_desc_sw128(v0 + kk * 16 * 128, C::CHUNK_BYTES, 1024), idesc_o, (jp | kk) != 0);
+          }
+          mma_commit(&v_empty[st]);
+          mma_commit(pv_done);
+        }
+      }
+    }
+  } else if (warp >= 4) {  // ---------------------------------------- softmax
+    const int q = warp & 3;
+    const int r = q * 32 + lane;                      // query row within the tile == TMEM lane
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkv; ++j) {
+      const int sb = j & 1;
+      if (!mbar_wait(&s_full[sb], (j >> 1) & 1)) { ok = false; break; }
+      tc_fence_after();
+      float s[kBKV];
+#pragma unroll
+      for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(tmem + lane_base + sb * kBKV + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
+      tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(&s_free[sb]);
+      const int64_t kv0 = (int64_t)j * kBKV;
+      float mx = -INFINITY;
+      if (kv0 + kBKV <= a.nk) {
+#pragma unroll
+        for (int i = 0; i < kBKV; ++i) {
+          s[i] *= a.scale_log2;
+          mx = fmaxf(mx, s[i]);
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < kBKV; ++i) {
+          s[i] = (kv0 + i < a.nk) ? s[i] * a.scale_log2 : -INFINITY;
+          mx = fmaxf(mx, s[i]);
+        }
+      }
+      if (j > 0) {
+        // PV_{j-1} must be done before O is rescaled or the P buffer reused
+        if (!mbar_wait(pv_done, (j - 1) & 1)) { ok = false; break; }
+        tc_fence_after();
+        const bool resc = mx > m_run + kRescaleLog2;
+        if (__any_sync(0xffffffffu, resc)) {
+          const float f = resc ? ex2_approx(m_run - mx) : 1.0f;
+#pragma unroll 1
+          for (int c = 0; c < D; c += 32) {
+            uint32_t o[32];
+            tmem_ld32(tmem + lane_base + C::O_COL + c, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+            tmem_st32(tmem + lane_base + C::O_COL + c, o);
+          }
+          tmem_wait_st();
+          if (resc) {
+            l_run *= f;
+            m_run = mx;
+          }
+        }
+      } else {
+        m_run = mx;
+      }
+      // P = 2^(s - m_run), stored as bf16 in the 128-byte-swizzled K-major layout
+      float ls = 0.f;
+#pragma unroll
+      for (int c8 = 0; c8 < kBKV / 8; ++c8) {
+        float p[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          p[i] = ex2_approx(s[c8 * 8 + i] - m_run);
+          ls += p[i];
+        }
+        uint4 u;
+        u.x = pack_bf16(p[0], p[1]);
+        u.y = pack_bf16(p[2], p[3]);
+        u.z = pack_bf16(p[4], p[5]);
+        u.w = pack_bf16(p[6], p[7]);
+        const int chunk = c8 >> 3, unit = c8 & 7;
+        *reinterpret_cast<uint4*>(sP + chunk * C::CHUNK_BYTES + r * 128 + ((unit ^ (r & 7)) << 4)) = u;
+      }
+      l_run += ls;
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(p_full);
+    }
+    // ---------------------------------------------------- epilogue: O / l
+    if (ok) ok = mbar_wait(pv_done, (nkv - 1) & 1);
+    tc_fence_after();
+    const int64_t row = (int64_t)qt * kBQ + r;
+    const float inv = 1.0f / l_run;
+#pragma unroll 1
+    for (int c = 0; c < D; c += 32) {
+      uint32_t o[32];
+      tmem_ld32(tmem + lane_base + C::O_COL + c, o);
+      tmem_wait_ld();
+      if (ok && row < a.nq) {
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]) * inv;
+        __nv_bfloat16* op = static_cast<__nv_bfloat16*>(a.out) + row * a.ldo + a.o_col + h * D + c;
+#pragma unroll
+        for (int i = 0; i < 32; i += 8) store8(op + i, v + i);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int D>
+acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
+  using C = AttnCfg<D>;
+  static bool attr_done = false;
+  if (!attr_done) {
+    ACID_CUDA(cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    attr_done = true;
+  }
+  CUtensorMap tq, tk, tv;
+  ACID_TRY(make_tmap_bf16(&tq, x.q, x.nq, x.ldq, x.ldq, kBQ));
+  ACID_TRY(make_tmap_bf16(&tk, x.k, x.nk, x.ldk, x.ldk, kBKV));
+  ACID_TRY(make_tmap_bf16(&tv, x.v, x.nk, x.ldv, x.ldv, kBKV));
+  AttnDev a;
+  a.nq = x.nq;
+  a.nk = x.nk;
+  a.q_col = x.q_col;
+  a.k_col = x.k_col;
+  a.v_col = x.v_col;
+  a.out = x.out;
+  a.ldo = x.ldo;
+  a.o_col = x.o_col;
+  a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
+  dim3 grid((unsigned)((x.nq + kBQ - 1) / kBQ), (unsigned)x.heads);
+  ProfScope prof(PROF_ATTENTION, 4.0 * (double)x.nq * (double)x.nk * D * x.heads, s);
+  attn_tc_kernel<D><<<grid, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+// ---------------------------------------------------------------- fp32 path
+__global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__ q, int64_t ldq, int q_col,
+                                                       const float* __restrict__ k, int64_t ldk, int k_col,
+                                                       const float* __restrict__ v, int64_t ldv, int v_col, float* out,
+                                                       int64_t ldo, int o_col, int64_t nq, int64_t nk, int D,
+                                                       float scale) {
+  const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int h = blockIdx.y;
+  const int lane = threadIdx.x & 31;
+  if (row >= nq) return;
+  constexpr int kMaxPer = 4;  // D <= 128
+  float qv[kMaxPer], o[kMaxPer];
+  const int per = D / 32;
+#pragma unroll
+  for (int i = 0; i < kMaxPer; ++i) {
+    qv[i] = i < per ? q[row * ldq + q_col + h * D + i * 32 + lane] : 0.f;
+    o[i] = 0.f;
+  }
+  float m = -INFINITY, l = 0.f;
+  for (int64_t j = 0; j < nk; ++j) {
+    const float* kr = k + j * ldk + k_col + h * D;
+    float sdot = 0.f;
+#pragma unroll
+    for (int i = 0; i < kMaxPer; ++i)
+      if (i < per) sdot = fmaf(qv[i], kr[i * 32 + lane], sdot);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sdot += __shfl_xor_sync(0xffffffffu, sdot, off);
+    const float sc = sdot * scale;
+    const float mn = fmaxf(m, sc);
+    const float corr = expf(m - mn);
+    const float p = expf(sc - mn);
+    l = l * corr + p;
+    const float* vr = v + j * ldv + v_col + h * D;
+#pragma unroll
+    for (int i = 0; i < kMaxPer; ++i)
+      if (i < per) o[i] = fmaf(p, vr[i * 32 + lane], o[i] * corr);
+    m = mn;
+  }
+#pragma unroll
+  for (int i = 0; i < kMaxPer; ++i)
+    if (i < per) out[row * ldo + o_col + h * D + i * 32 + lane] = o[i] / l;
+}
+
+}  // namespace
+
+acid_status attention_forward(int dtype, const AttnArgs& x, cudaStream_t s) {
+  ACID_REQUIRE(x.q && x.k && x.v && x.out, ACID_ERR_INVALID_ARG, "attention: null pointer");
+  ACID_REQUIRE(x.nk > 0 && x.nq >= 0 && x.heads > 0, ACID_ERR_INVALID_ARG, "attention: bad shape");
+  if (x.nq == 0) return ACID_OK;
+  if (dtype == ACID_FP32) {
+    ACID_REQUIRE(x.head_dim % 32 == 0 && x.head_dim <= 128, ACID_ERR_UNSUPPORTED,
+                 "attention fp32: head_dim must be 32, 64, 96 or 128");
+    dim3 grid((unsigned)((x.nq + 7) / 8), (unsigned)x.heads);
+    attn_f32_kernel<<<grid, 256, 0, s>>>((const float*)x.q, x.ldq, x.q_col, (const float*)x.k, x.ldk, x.k_col,
+                                         (const float*)x.v, x.ldv, x.v_col, (float*)x.out, x.ldo, x.o_col, x.nq, x.nk,
+                                         x.head_dim, (float)(1.0 / sqrt((double)x.head_dim)));
+    ACID_CHECK_LAUNCH();
+    return ACID_OK;
+  }
+  ACID_REQUIRE(x.head_dim == 64 || x.head_dim == 128, ACID_ERR_UNSUPPORTED, "attention bf16: head_dim must be 64 or 128");
+  ACID_REQUIRE(x.q_col % 8 == 0 && x.k_col % 8 == 0 && x.v_col % 8 == 0 && x.o_col % 8 == 0 && x.ldo % 8 == 0,
+               ACID_ERR_UNSUPPORTED, "attention bf16: column offsets must be multiples of 8");
+  ACID_REQUIRE(aligned(x.out, 16), ACID_ERR_UNSUPPORTED, "attention bf16: output must be 16-byte aligned");
+  if (x.head_dim == 128) return launch_attn_tc<128>(x, s);
+  return launch_attn_tc<64>(x, s);
+}
+
+ACID_DEVICE_FLAG_READER(take_device_error_attention)
+
+}  // namespace acid

@@ -1,0 +1,413 @@
+// Linear layers of the DiT block.
+//
+// bf16: a tcgen05 GEMM.  One CTA computes a 128 x BN output tile with the
+// fp32 accumulator in tensor memory (TMEM).  Warp 0 streams 128x64 A and
+// BNx64 B tiles with TMA (128-byte swizzle) through a STAGES-deep mbarrier
+// ring; warp 1 issues tcgen05.mma (M=128, N=BN, K=16) from one thread;
+// warps 2-5 wait for the accumulator, read it back with tcgen05.ld (one
+// thread per output row) and apply the fused epilogue (bias, GELU-tanh,
+// 3D RoPE of q/k, gated or plain residual) before storing.
+//
+// fp32: a register-tiled SIMT GEMM with the same epilogue (the fp32 mode's
+// 1e-4 tolerance rules out tf32 tensor cores).
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace acid {
+
+namespace {
+
+// Epilogue parameters as passed to the kernels.
+struct EpiDev {
+  int kind;
+  const float* bias;
+  const float* gate_v;
+  const float* gate_t;
+  int64_t gate_split;
+  const void* res;
+  int64_t ldr;
+  int64_t row_base;
+  RopeTable rope;
+  int64_t rope_first_video;
+  int d, head_dim;
+};
+
+EpiDev to_dev(const Epilogue& e) {
+  EpiDev d;
+  d.kind = e.kind;
+  d.bias = e.bias;
+  d.gate_v = e.gate_video;
+  d.gate_t = e.gate_text ? e.gate_text : e.gate_video;
+  d.gate_split = e.gate_split;
+  d.res = e.residual;
+  d.ldr = e.ldr;
+  d.row_base = e.row_base;
+  d.rope = e.rope;
+  d.rope_first_video = e.rope_first_video;
+  d.d = e.d;
+  d.head_dim = e.head_dim;
+  return d;
+}
+
+// (cos, sin) of the RoPE angle of pair `jj` (within the head) at video position pos.
+__device__ __forceinline__ float2 rope_cs(const RopeTable& t, int64_t pos, int jj) {
+  const int64_t hw = (int64_t)t.grid_h * t.grid_w;
+  const int f = (int)(pos / hw);
+  const int h = (int)((pos / t.grid_w) % t.grid_h);
+  const int w = (int)(pos % t.grid_w);
+  if (jj < t.pairs_t) return t.table[(int64_t)f * t.pairs_t + jj];
+  jj -= t.pairs_t;
+  const int64_t off_h = (int64_t)t.grid_f * t.pairs_t;
+  if (jj < t.pairs_h) return t.table[off_h + (int64_t)h * t.pairs_h + jj];
+  jj -= t.pairs_h;
+  const int64_t off_w = off_h + (int64_t)t.grid_h * t.pairs_h;
+  return t.table[off_w + (int64_t)w * t.pairs_w + jj];
+}
+
+// Applies the epilogue to the adjacent outputs (grow, col) and (grow, col+1).
+// r0/r1: residual values (read by the caller) for the residual kinds.
+template <bool kFastGelu>
+__device__ __forceinline__ void epi_pair(const EpiDev& e, int64_t grow, int col, float& a, float& b, float r0,
+                                         float r1) {
+  if (e.bias) {
+    a += e.bias[col];
+    b += e.bias[col + 1];
+  }
+  switch (e.kind) {
+    case EPI_GELU:
+      a = gelu_tanh<kFastGelu>(a);
+      b = gelu_tanh<kFastGelu>(b);
+      break;
+    case EPI_ROPE_QKV:
+      if (col < 2 * e.d && grow >= e.rope_first_video) {
+        const float2 cs = rope_cs(e.rope, grow - e.rope_first_video, (col % e.head_dim) >> 1);
+        const float x0 = a, x1 = b;
+        a = x0 * cs.x - x1 * cs.y;
+        b = x0 * cs.y + x1 * cs.x;
+      }
+      break;
+    case EPI_GATED_RES: {
+      const float* g = grow < e.gate_split ? e.gate_t : e.gate_v;
+      a = fmaf(g[col], a, r0);
+      b = fmaf(g[col + 1], b, r1);
+      break;
+    }
+    case EPI_RES:
+      a += r0;
+      b += r1;
+      break;
+    default:
+      break;
+  }
+}
+
+__host__ __device__ __forceinline__ bool epi_reads_res(int kind) { return kind == EPI_GATED_RES || kind == EPI_RES; }
+
+// ===========================================================================
+// tcgen05 GEMM (bf16 in, fp32 accumulate)
+// ===========================================================================
+constexpr int BM = 128, BK = 64;
+constexpr int kGemmThreads = 192;
+
+template <int BN>
+struct TcCfg {
+  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+};
+
+struct GemmDims {
+  int64_t M;
+  int N, K;
+  void* out;
+  int64_t ldo;
+  int out_fp32;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
+                   EpiDev e) {
+  using C = TcCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* accum = empty + C::STAGES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_tile = blockIdx.x, m_tile = blockIdx.y;
+  const int num_kb = (g.K + BK - 1) / BK;
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, BN);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // TMA producer
+      for (int kb = 0; kb < num_kb; ++kb) {
+        const int s = kb % C::STAGES, round = kb / C::STAGES;
+        if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1)) break;
+        mbar_expect_tx(&full[s], C::STAGE_BYTES);
+        tma_load_2d(sA + s * C::A_BYTES, &tmA, &full[s], kb * BK, m_tile * BM);
+        tma_load_2d(sB + s * C::B_BYTES, &tmB, &full[s], kb * BK, n_tile * BN);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // MMA issuer
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
+      bool ok = true;
+      for (int kb = 0; kb < num_kb && ok; ++kb) {
+        const int s = kb % C::STAGES, round = kb / C::STAGES;
+        if (!mbar_wait(&full[s], round & 1)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+        const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k) {
+          const uint64_t ad = smem_desc_sw128(a0 + k * 32, 16, 1024);
+          const uint64_t bd = smem_desc_sw128(b0 + k * 32, 16, 1024);
+          mma_bf16_ss(tmem, ad, bd, idesc, (kb | k) != 0);
+        }
+        mma_commit(&empty[s]);
+      }
+      if (ok) mma_commit(accum);
+    }
+  } else {  // epilogue: warps 2..5 -> TMEM lane quarters 2, 3, 0, 1
+    const int q = warp & 3;
+    const bool ok = mbar_wait(accum, 0);
+    tc_fence_after();
+    const int64_t row = (int64_t)m_tile * BM + q * 32 + lane;
+    const int64_t grow = row + e.row_base;
+    const bool row_ok = ok && row < g.M;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
+      tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + c, r);
+      tmem_wait_ld();
+      const int col0 = n_tile * BN + c;
+      if (!row_ok || col0 >= g.N) continue;
+      float v[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+      float rv[32];
+      if (epi_reads_res(e.kind)) {
+        if (g.out_fp32) {
+          const float* rp = static_cast<const float*>(e.res) + row * e.ldr + col0;
+#pragma unroll
+          for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
+        } else {
+          const __nv_bfloat16* rp = static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col0;
+#pragma unroll
+          for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) rv[j] = 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 32; j += 2) epi_pair<true>(e, grow, col0 + j, v[j], v[j + 1], rv[j], rv[j + 1]);
+      if (g.out_fp32) {
+        float* op = static_cast<float*>(g.out) + row * g.ldo + col0;
+#pragma unroll
+        for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
+      } else {
+        __nv_bfloat16* op = static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col0;
+#pragma unroll
+        for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, BN);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// TMA descriptor encoding through the driver entry point (no -lcuda needed)
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+}  // namespace
+
+// Row-major bf16 matrix [rows, cols] with row stride ld (elements), boxes of
+// box_rows x 64 columns, 128-byte swizzle, zero fill out of bounds.
+acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+  auto fn = encode_fn();
+  ACID_REQUIRE(fn != nullptr, ACID_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  ACID_REQUIRE(aligned(base, 16) && (ld * 2) % 16 == 0, ACID_ERR_UNSUPPORTED,
+               "TMA operand must be 16-byte aligned with a row stride that is a multiple of 8 elements");
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1u, 1u};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  ACID_REQUIRE(r == CUDA_SUCCESS, ACID_ERR_CUDA, "cuTensorMapEncodeTiled failed (code " + std::to_string((int)r) + ")");
+  return ACID_OK;
+}
+
+namespace {
+
+template <int BN>
+acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
+                      const Epilogue& epi, cudaStream_t s) {
+  using C = TcCfg<BN>;
+  static bool attr_done = false;
+  if (!attr_done) {
+    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    attr_done = true;
+  }
+  CUtensorMap ta, tb;
+  ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
+  ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, BN));
+  GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0};
+  dim3 grid((N + BN - 1) / BN, (unsigned)((M + BM - 1) / BM));
+  ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
+  gemm_tc_kernel<BN><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+// ===========================================================================
+// fp32 SIMT GEMM: 64x64 tile, 16-deep K slices, 4x4 outputs per thread
+// ===========================================================================
+constexpr int SB = 64, SK = 16;
+
+template <typename TW>
+__global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__ A, int64_t lda, int64_t M, int K,
+                                                       const TW* __restrict__ W, int N, float* out, int64_t ldo,
+                                                       EpiDev e) {
+  __shared__ float As[SK][SB + 4];
+  __shared__ float Ws[SK][SB + 4];
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  const int64_t m0 = (int64_t)blockIdx.y * SB;
+  const int n0 = blockIdx.x * SB;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < K; k0 += SK) {
+    for (int i = threadIdx.x; i < SB * SK; i += 256) {
+      const int r = i / SK, kk = i % SK;
+      const int64_t gm = m0 + r;
+      const int gk = k0 + kk, gn = n0 + r;
+      As[kk][r] = (gm < M && gk < K) ? A[gm * lda + gk] : 0.f;
+      Ws[kk][r] = (gn < N && gk < K) ? io<TW>::ld(W + (int64_t)gn * K + gk) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < SK; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        a[i] = As[kk][ty * 4 + i];
+        b[i] = Ws[kk][tx * 4 + i];
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  const float* res = static_cast<const float*>(e.res);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t row = m0 + ty * 4 + i;
+    if (row >= M) continue;
+    const int64_t grow = row + e.row_base;
+#pragma unroll
+    for (int j = 0; j < 4; j += 2) {
+      const int col = n0 + tx * 4 + j;
+      if (col >= N) continue;  // N is even
+      float r0 = 0.f, r1 = 0.f;
+      if (epi_reads_res(e.kind)) {
+        r0 = res[row * e.ldr + col];
+        r1 = res[row * e.ldr + col + 1];
+      }
+      float a = acc[i][j], b = acc[i][j + 1];
+      epi_pair<false>(e, grow, col, a, b, r0, r1);
+      out[row * ldo + col] = a;
+      out[row * ldo + col + 1] = b;
+    }
+  }
+}
+
+}  // namespace
+
+acid_status linear_forward_f32(const void* A, int64_t lda, int64_t M, int K, int w_dtype, const void* W, int N,
+                               void* out, int64_t ldo, const Epilogue& epi, cudaStream_t s) {
+  ACID_REQUIRE(A && W && out, ACID_ERR_INVALID_ARG, "linear: null pointer");
+  ACID_REQUIRE(M >= 0 && K > 0 && N > 0, ACID_ERR_INVALID_ARG, "linear: bad shape");
+  ACID_REQUIRE(N % 2 == 0, ACID_ERR_UNSUPPORTED, "linear fp32: N must be even");
+  if (M == 0) return ACID_OK;
+  dim3 grid((N + SB - 1) / SB, (unsigned)((M + SB - 1) / SB));
+  if (w_dtype == ACID_BF16)
+    gemm_f32_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const float*>(A), lda, M, K,
+                                                        static_cast<const __nv_bfloat16*>(W), N,
+                                                        static_cast<float*>(out), ldo, to_dev(epi));
+  else
+    gemm_f32_kernel<float><<<grid, 256, 0, s>>>(static_cast<const float*>(A), lda, M, K,
+                                                static_cast<const float*>(W), N, static_cast<float*>(out), ldo,
+                                                to_dev(epi));
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out,
+                           int64_t ldo, const Epilogue& epi, cudaStream_t s) {
+  ACID_REQUIRE(A && W && out, ACID_ERR_INVALID_ARG, "linear: null pointer");
+  ACID_REQUIRE(M >= 0 && K > 0 && N > 0, ACID_ERR_INVALID_ARG, "linear: bad shape");
+  if (M == 0) return ACID_OK;
+  ACID_REQUIRE(epi.kind != EPI_ROPE_QKV || (epi.rope.table != nullptr && epi.head_dim > 0 && epi.d > 0),
+               ACID_ERR_INVALID_ARG, "linear: RoPE epilogue needs a table");
+  ACID_REQUIRE(!epi_reads_res(epi.kind) || epi.residual != nullptr, ACID_ERR_INVALID_ARG,
+               "linear: residual epilogue needs a residual");
+  if (dtype == ACID_FP32) return linear_forward_f32(A, lda, M, K, ACID_FP32, W, N, out, ldo, epi, s);
+  ACID_REQUIRE(N % 32 == 0 && K % 8 == 0, ACID_ERR_UNSUPPORTED, "linear bf16: need N % 32 == 0 and K % 8 == 0");
+  ACID_REQUIRE(ldo % 8 == 0 && aligned(out, 16) && (!epi.residual || (epi.ldr % 8 == 0 && aligned(epi.residual, 16))),
+               ACID_ERR_UNSUPPORTED, "linear bf16: output/residual must be 16-byte aligned rows");
+  if (N % 256 == 0) return launch_tc<256>(A, lda, M, K, W, N, out, ldo, epi, s);
+  if (N % 128 == 0) return launch_tc<128>(A, lda, M, K, W, N, out, ldo, epi, s);
+  return launch_tc<64>(A, lda, M, K, W, N, out, ldo, epi, s);
+}
+
+ACID_DEVICE_FLAG_READER(take_device_error_gemm)
+
+}  // namespace acid

@@ -1,0 +1,413 @@
+// The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler flow-matching
+// sampler, with TeaCache or EasyCache (Sec. 2) as the wrapped method.  All
+// tensor work runs in the library's kernels; the host keeps only the scalar
+// controller state and takes one decision per non-warmup step from the drift
+// value it reads back.
+#include <math.h>
+#include <string.h>
+
+#include <string>
+
+#include "block.h"
+#include "common.cuh"
+#include "internal.h"
+
+namespace acid {
+
+namespace {
+
+size_t es(int dt) { return dt == ACID_BF16 ? 2 : 4; }
+
+struct LoopWs {
+  float* sinus;
+  float* temb_h;
+  float* temb;
+  float* mod0;      // block 0 shift / scale (TEMNI)
+  float* fmod;      // final layer shift / scale
+  uint8_t* tokens;  // [N, P] fp32 patch vectors
+  float* h_in;      // [N, d] patch embedding (fp32)
+  float* temni[2];  // [N, d] block-0 modulated input, current / previous
+  float* resid;     // [N, d] TeaCache residual H_out - H_in
+  uint8_t* xbuf;    // [L + N, d] block-stack state (model dtype)
+  uint8_t* text;    // [L, d] text context / text tokens (model dtype)
+  uint8_t* y;       // [N, d] final LayerNorm output
+  float* vtok;      // [N, P] final layer output
+  float* v[2];      // latent-sized velocity, current / previous (EasyCache)
+  float* x_prev;    // latent-sized previous input (EasyCache)
+  float* offset;    // latent-sized v_c - x_c (EasyCache)
+  double* dres;     // [8] device drift results
+  uint8_t* drift_ws;
+  float2* rope;
+  uint8_t* block_base;
+  size_t bytes;
+};
+
+struct Shape {
+  int64_t N, L, P, latent;
+  int d;
+};
+
+Shape shape_of(const acid_model& m) {
+  Shape s;
+  const int64_t gf = m.latent_f / m.pt, gh = m.latent_h / m.ph, gw = m.latent_w / m.pw;
+  s.N = gf * gh * gw;
+  s.L = m.block.n_text;
+  s.P = (int64_t)m.latent_c * m.pt * m.ph * m.pw;
+  s.latent = (int64_t)m.latent_c * m.latent_f * m.latent_h * m.latent_w;
+  s.d = m.block.d;
+  return s;
+}
+
+acid_block_desc desc_for(const acid_model& m, int i) {
+  acid_block_desc d = m.block;
+  if (m.block.kind == ACID_BLOCK_HV_DUAL || m.block.kind == ACID_BLOCK_HV_SINGLE)
+    d.kind = i < m.n_blocks ? ACID_BLOCK_HV_DUAL : ACID_BLOCK_HV_SINGLE;
+  return d;
+}
+
+int total_blocks(const acid_model& m) {
+  const bool hv = m.block.kind == ACID_BLOCK_HV_DUAL || m.block.kind == ACID_BLOCK_HV_SINGLE;
+  return m.n_blocks + (hv ? m.n_single : 0);
+}
+
+LoopWs loop_layout(const acid_model& m, void* base) {
+  Bump b{static_cast<uint8_t*>(base)};
+  const Shape s = shape_of(m);
+  const int dt = m.block.dtype;
+  LoopWs w;
+  w.sinus = b.take<float>(m.time_freq_dim);
+  w.temb_h = b.take<float>(s.d);
+  w.temb = b.take<float>(s.d);
+  w.mod0 = b.take<float>(2 * s.d);
+  w.fmod = b.take<float>(2 * s.d);
+  w.tokens = b.take<uint8_t>(s.N * s.P * sizeof(float));
+  w.h_in = b.take<float>(s.N * s.d);
+  w.temni[0] = b.take<float>(s.N * s.d);
+  w.temni[1] = b.take<float>(s.N * s.d);
+  w.resid = b.take<float>(s.N * s.d);
+  const int64_t xrows = m.block.kind == ACID_BLOCK_WAN ? s.N : s.N + s.L;
+  w.xbuf = b.take<uint8_t>(xrows * s.d * es(dt));
+  w.text = b.take<uint8_t>(std::max<int64_t>(s.L, 1) * s.d * es(dt));
+  w.y = b.take<uint8_t>(s.N * s.d * es(dt));
+  w.vtok = b.take<float>(s.N * s.P);
+  w.v[0] = b.take<float>(s.latent);
+  w.v[1] = b.take<float>(s.latent);
+  w.x_prev = b.take<float>(s.latent);
+  w.offset = b.take<float>(s.latent);
+  w.dres = b.take<double>(8);
+  w.drift_ws = b.take<uint8_t>(drift_workspace_bytes(0));
+  RopeTable rt = rope_layout(m.block.grid_f, m.block.grid_h, m.block.grid_w, m.block.d / std::max(1, m.block.heads));
+  w.rope = b.take<float2>((size_t)rt.elems());
+  // one block workspace, sized for the larger of the first and last block kinds
+  size_t blk = block_ws_layout(desc_for(m, 0), nullptr).bytes;
+  blk = std::max(blk, block_ws_layout(desc_for(m, total_blocks(m) - 1), nullptr).bytes);
+  w.block_base = b.take<uint8_t>(blk);
+  w.bytes = b.off + 1024;
+  return w;
+}
+
+acid_status validate_model(const acid_model& m) {
+  ACID_REQUIRE(m.blocks != nullptr && m.n_blocks > 0, ACID_ERR_INVALID_ARG, "model: no blocks");
+  ACID_TRY(validate_block_desc(m.block));
+  ACID_REQUIRE(m.latent_c > 0 && m.pt > 0 && m.ph > 0 && m.pw > 0 && m.latent_f % m.pt == 0 &&
+                   m.latent_h % m.ph == 0 && m.latent_w % m.pw == 0,
+               ACID_ERR_INVALID_ARG, "model: latent shape not divisible by the patch size");
+  ACID_REQUIRE(m.block.grid_f == m.latent_f / m.pt && m.block.grid_h == m.latent_h / m.ph &&
+                   m.block.grid_w == m.latent_w / m.pw,
+               ACID_ERR_INVALID_ARG, "model: block grid does not match latent / patch");
+  ACID_REQUIRE(m.time_freq_dim > 0 && m.time_freq_dim % 16 == 0, ACID_ERR_INVALID_ARG,
+               "model: time_freq_dim must be a positive multiple of 16");
+  ACID_REQUIRE(m.patch.w && m.time1.w && m.time2.w && m.final_mod.w && m.final_out.w, ACID_ERR_INVALID_ARG,
+               "model: missing patch / time / final weights");
+  const int64_t P = (int64_t)m.latent_c * m.pt * m.ph * m.pw;
+  ACID_REQUIRE(P % 64 == 0 || m.block.dtype == ACID_FP32, ACID_ERR_UNSUPPORTED,
+               "model bf16: patch dimension C*pt*ph*pw must be a multiple of 64");
+  if (m.block.kind == ACID_BLOCK_WAN && m.block.n_text > 0)
+    ACID_REQUIRE(m.text.w != nullptr && m.d_text > 0 && m.d_text % 64 == 0, ACID_ERR_INVALID_ARG,
+                 "model: WAN with text needs the text projection (d_text % 64 == 0)");
+  if (m.block.kind != ACID_BLOCK_WAN)
+    ACID_REQUIRE(m.d_text == m.block.d || m.block.n_text == 0, ACID_ERR_INVALID_ARG,
+                 "model: joint text tokens must be given at width d");
+  for (int i = 0; i < total_blocks(m); ++i) ACID_TRY(validate_block_weights(desc_for(m, i), m.blocks[i]));
+  return ACID_OK;
+}
+
+acid_status validate_cfg(const acid_loop_cfg& c) {
+  ACID_REQUIRE(c.n_steps > 0 && c.warmup >= 0, ACID_ERR_INVALID_ARG, "loop: n_steps must be > 0, warmup >= 0");
+  ACID_REQUIRE(c.method == ACID_METHOD_TEACACHE || c.method == ACID_METHOD_EASYCACHE, ACID_ERR_INVALID_ARG,
+               "loop: unknown method");
+  ACID_REQUIRE(c.method != ACID_METHOD_EASYCACHE || c.warmup >= 2, ACID_ERR_INVALID_ARG,
+               "loop: EasyCache needs warmup >= 2 (k is defined after two computed steps)");
+  ACID_REQUIRE(c.shift > 0.0, ACID_ERR_INVALID_ARG, "loop: shift must be > 0");
+  return ACID_OK;
+}
+
+double sigma_at(const acid_loop_cfg& c, int i) {
+  const double s = 1.0 - (double)i / c.n_steps;
+  if (c.shift == 1.0) return s;
+  return c.shift * s / (1.0 + (c.shift - 1.0) * s);
+}
+
+// Algorithm 1, the non-warmup branch: accumulate, pick the threshold from the
+// signal's rate of change, compare, reset on compute; s_prev always updated.
+bool controller_step(acid_loop_state& st, const acid_loop_cfg& c, double s, int forced, acid_step_log* lg) {
+  st.sigma_acc += s;
+  double tau, ds = NAN;
+  if (st.have_prev_signal) {
+    ds = fabs(s - st.s_prev);
+    tau = ds <= c.delta ? c.tau_high : c.tau_low;
+  } else {
+    tau = c.tau_low;
+  }
+  const double seen = st.sigma_acc;
+  bool skip = seen <= tau;
+  if (forced >= 0) skip = forced == 0;
+  if (!skip) st.sigma_acc = 0.0;
+  st.s_prev = s;
+  st.have_prev_signal = 1;
+  if (lg) {
+    lg->signal = s;
+    lg->dsignal = ds;
+    lg->tau = tau;
+    lg->sigma = seen;
+    lg->forced = forced >= 0;
+  }
+  return !skip;
+}
+
+double ratio_or_inf(double num, double den) {
+  if (den == 0.0) return num == 0.0 ? 0.0 : INFINITY;
+  return num / den;
+}
+
+acid_status read_results(double* host, const double* dev, int n, cudaStream_t s) {
+  ACID_CUDA(cudaMemcpyAsync(host, dev, sizeof(double) * n, cudaMemcpyDeviceToHost, s));
+  ACID_CUDA(cudaStreamSynchronize(s));
+  return ACID_OK;
+}
+
+// Runs every block on the state in w.xbuf.
+acid_status run_blocks(const acid_model& m, const LoopWs& w, cudaStream_t s) {
+  const RopeTable base_rope = [&] {
+    RopeTable t = rope_layout(m.block.grid_f, m.block.grid_h, m.block.grid_w, m.block.d / m.block.heads);
+    t.table = w.rope;
+    return t;
+  }();
+  const void* ctx = m.block.kind == ACID_BLOCK_WAN && m.block.n_text > 0 ? w.text : nullptr;
+  for (int i = 0; i < total_blocks(m); ++i) {
+    const acid_block_desc d = desc_for(m, i);
+    const BlockWs bws = block_ws_layout(d, w.block_base);
+    ACID_TRY(block_forward_impl(d, w.xbuf, w.temb, ctx, m.blocks[i], bws, &base_rope, s));
+  }
+  return ACID_OK;
+}
+
+// Final layer + unpatchify: v (optional) and the Euler update of the latent.
+acid_status final_layer(const acid_model& m, const LoopWs& w, const void* h_out, float* v_out, float* latent,
+                        float dsig, cudaStream_t s) {
+  const Shape sh = shape_of(m);
+  const int dt = m.block.dtype;
+  ACID_TRY(gemv(dt, m.final_mod.w, m.final_mod.b, w.temb, w.fmod, 2 * sh.d, sh.d, true, s));
+  ACID_TRY(ln_mod(dt, h_out, dt, w.y, sh.N, sh.d, w.fmod, w.fmod + sh.d, nullptr, nullptr, 0, m.block.ln_eps, s));
+  Epilogue e;
+  e.bias = m.final_out.b;
+  e.out_fp32 = true;
+  ACID_TRY(linear_forward(dt, w.y, sh.d, sh.N, sh.d, m.final_out.w, (int)sh.P, w.vtok, sh.P, e, s));
+  return unpatchify_euler(w.vtok, v_out, latent, m.latent_c, m.latent_f, m.latent_h, m.latent_w, m.pt, m.ph, m.pw,
+                          dsig, s);
+}
+
+}  // namespace
+
+}  // namespace acid
+
+using namespace acid;
+
+extern "C" acid_status acid_loop_workspace_size(const acid_model* m, size_t* bytes) {
+  clear_error();
+  ACID_REQUIRE(m && bytes, ACID_ERR_INVALID_ARG, "acid_loop_workspace_size: null argument");
+  ACID_TRY(validate_model(*m));
+  *bytes = loop_layout(*m, nullptr).bytes;
+  return ACID_OK;
+}
+
+static acid_status check_ws(const acid_model& m, void* ws, size_t bytes, LoopWs* out) {
+  ACID_REQUIRE(ws != nullptr && aligned(ws, 1024), ACID_ERR_WORKSPACE, "loop: workspace null or not 1024-aligned");
+  *out = loop_layout(m, ws);
+  ACID_REQUIRE(bytes >= out->bytes, ACID_ERR_WORKSPACE,
+               "loop: workspace too small (need " + std::to_string(out->bytes) + " bytes)");
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_loop_begin(const acid_model* m, const acid_loop_cfg* cfg, const void* text,
+                                       acid_loop_state* state, void* workspace, size_t workspace_bytes,
+                                       acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m && cfg && state, ACID_ERR_INVALID_ARG, "acid_loop_begin: null argument");
+  ACID_TRY(validate_model(*m));
+  ACID_TRY(validate_cfg(*cfg));
+  LoopWs w;
+  ACID_TRY(check_ws(*m, workspace, workspace_bytes, &w));
+  cudaStream_t s = (cudaStream_t)stream;
+  memset(state, 0, sizeof(*state));
+  const Shape sh = shape_of(*m);
+  const int dt = m->block.dtype;
+  if (sh.L > 0) {
+    ACID_REQUIRE(text != nullptr && aligned(text, 16), ACID_ERR_INVALID_ARG,
+                 "acid_loop_begin: text must be a 16-byte aligned device pointer");
+    if (m->block.kind == ACID_BLOCK_WAN) {
+      Epilogue e;
+      e.bias = m->text.b;
+      ACID_TRY(linear_forward(dt, text, m->d_text, sh.L, m->d_text, m->text.w, sh.d, w.text, sh.d, e, s));
+    } else {
+      ACID_CUDA(cudaMemcpyAsync(w.text, text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
+    }
+  }
+  RopeTable rt = rope_layout(m->block.grid_f, m->block.grid_h, m->block.grid_w, m->block.d / m->block.heads);
+  ACID_TRY(rope_build(rt, w.rope, m->block.rope_theta, s));
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cfg* cfg, acid_loop_state* st,
+                                         void* latent_v, acid_step_log* log, void* workspace, size_t workspace_bytes,
+                                         acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m && cfg && st && latent_v, ACID_ERR_INVALID_ARG, "acid_denoise_step: null argument");
+  ACID_TRY(validate_cfg(*cfg));
+  ACID_REQUIRE(st->step >= 0 && st->step < cfg->n_steps, ACID_ERR_INVALID_ARG, "acid_denoise_step: step out of range");
+  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_denoise_step: latent must be 16-byte aligned");
+  LoopWs w;
+  ACID_TRY(check_ws(*m, workspace, workspace_bytes, &w));
+  cudaStream_t s = (cudaStream_t)stream;
+  float* latent = static_cast<float*>(latent_v);
+  const Shape sh = shape_of(*m);
+  const int dt = m->block.dtype;
+  const int i = st->step;
+  const double sig = sigma_at(*cfg, i), sig_next = sigma_at(*cfg, i + 1);
+  const double t = 1000.0 * sig;
+  const float dsig = (float)(sig_next - sig);
+  const bool warm = i < cfg->warmup;
+  int forced = cfg->forced ? cfg->forced[i] : -1;
+  if (forced < 0 && cfg->force_last && i == cfg->n_steps - 1) forced = 1;
+
+  acid_step_log lg;
+  memset(&lg, 0, sizeof(lg));
+  lg.step = i;
+  lg.warmup = warm;
+  lg.t = t;
+  lg.signal = lg.dsignal = lg.tau = lg.sigma = NAN;
+  cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+  if (log) {
+    ACID_CUDA(cudaEventCreate(&ev0));
+    ACID_CUDA(cudaEventCreate(&ev1));
+    ACID_CUDA(cudaEventRecord(ev0, s));
+  }
+
+  // timestep embedding: temb = W2 SiLU(W1 sinusoid(t) + b1) + b2
+  ACID_TRY(timestep_sinusoid(w.sinus, t, m->time_freq_dim, s));
+  ACID_TRY(gemv(dt, m->time1.w, m->time1.b, w.sinus, w.temb_h, sh.d, m->time_freq_dim, false, s));
+  ACID_TRY(gemv(dt, m->time2.w, m->time2.b, w.temb_h, w.temb, sh.d, sh.d, true, s));
+  // patch embedding H_in (fp32)
+  // (fp32 tokens and accumulation: the drift signal compares consecutive H_in
+  // that differ by a few percent, so it must not see bf16 input rounding)
+  ACID_TRY(patchify(latent, ACID_FP32, w.tokens, m->latent_c, m->latent_f, m->latent_h, m->latent_w, m->pt, m->ph,
+                    m->pw, s));
+  {
+    Epilogue e;
+    e.bias = m->patch.b;
+    e.out_fp32 = true;
+    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m->patch.w, sh.d, w.h_in, sh.d, e, s));
+  }
+  const int64_t vrow0 = m->block.kind == ACID_BLOCK_WAN ? 0 : sh.L;
+  void* x_video = w.xbuf + vrow0 * sh.d * es(dt);
+  auto run_model = [&]() -> acid_status {
+    if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
+    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
+    return run_blocks(*m, w, s);
+  };
+
+  bool compute = true;
+  if (cfg->method == ACID_METHOD_TEACACHE) {
+    // s_t: rel_l1 of block 0's modulated input between consecutive steps
+    const int cur = i & 1, prv = cur ^ 1;
+    ACID_TRY(gemv(dt, m->blocks[0].mod.w, m->blocks[0].mod.b, w.temb, w.mod0, 2 * sh.d, sh.d, true, s));
+    ACID_TRY(ln_mod(ACID_FP32, w.h_in, ACID_FP32, w.temni[cur], sh.N, sh.d, w.mod0, w.mod0 + sh.d, nullptr, nullptr,
+                    0, m->block.ln_eps, s));
+    if (!warm) {
+      ACID_REQUIRE(i > 0, ACID_ERR_INVALID_ARG, "TeaCache needs at least one warmup step");
+      ACID_TRY(drift_launch(ACID_FP32, w.temni[prv], w.temni[cur], nullptr, nullptr, sh.N * sh.d, w.dres,
+                            w.drift_ws, drift_workspace_bytes(0), s));
+      double h[3];
+      ACID_TRY(read_results(h, w.dres, 3, s));
+      compute = controller_step(*st, *cfg, h[0], forced, &lg);
+    }
+    if (compute || !st->have_cache) {
+      compute = true;
+      ACID_TRY(run_model());
+      ACID_TRY(add_mixed(dt, x_video, ACID_FP32, w.h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s));
+      st->have_cache = 1;
+    } else {
+      ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s));
+    }
+    ACID_TRY(final_layer(*m, w, x_video, nullptr, latent, dsig, s));
+  } else {
+    // EasyCache: s_t = k mean|x_t - x_{t-1}| / mean|v_{t-1}|
+    float* v = w.v[i & 1];
+    float* v_prev = w.v[(i & 1) ^ 1];
+    if (!warm) {
+      ACID_REQUIRE(st->have_rate, ACID_ERR_INVALID_ARG, "EasyCache: transformation rate undefined");
+      ACID_TRY(drift_launch(ACID_FP32, w.x_prev, latent, nullptr, nullptr, sh.latent, w.dres, w.drift_ws,
+                            drift_workspace_bytes(0), s));
+      ACID_TRY(drift_launch(ACID_FP32, v_prev, v_prev, nullptr, nullptr, sh.latent, w.dres + 3, w.drift_ws,
+                            drift_workspace_bytes(0), s));
+      double h[6];
+      ACID_TRY(read_results(h, w.dres, 6, s));
+      const double sig_t = ratio_or_inf(st->k_rate * (h[1] / sh.latent), h[5] / sh.latent);
+      compute = controller_step(*st, *cfg, sig_t, forced, &lg);
+    }
+    if (compute || !st->have_cache) {
+      compute = true;
+      ACID_TRY(run_model());
+      ACID_TRY(final_layer(*m, w, x_video, v, nullptr, 0.0f, s));
+      if (i > 0) {  // k = mean|v_c - v_{c-1}| / mean|x_c - x_{c-1}|
+        ACID_TRY(drift_launch(ACID_FP32, v_prev, v, nullptr, nullptr, sh.latent, w.dres, w.drift_ws,
+                              drift_workspace_bytes(0), s));
+        ACID_TRY(drift_launch(ACID_FP32, w.x_prev, latent, nullptr, nullptr, sh.latent, w.dres + 3, w.drift_ws,
+                              drift_workspace_bytes(0), s));
+        double h[6];
+        ACID_TRY(read_results(h, w.dres, 6, s));
+        st->k_rate = ratio_or_inf(h[1] / sh.latent, h[4] / sh.latent);
+        st->have_rate = 1;
+      }
+      ACID_TRY(add_mixed(ACID_FP32, v, ACID_FP32, latent, ACID_FP32, w.offset, sh.latent, -1.0f, s));
+      st->have_cache = 1;
+    } else {
+      ACID_TRY(add_mixed(ACID_FP32, latent, ACID_FP32, w.offset, ACID_FP32, v, sh.latent, 1.0f, s));
+    }
+    ACID_CUDA(cudaMemcpyAsync(w.x_prev, latent, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
+    ACID_TRY(euler_update(latent, v, sh.latent, dsig, s));
+  }
+  lg.computed = compute;
+  st->step = i + 1;
+  if (log) {
+    ACID_CUDA(cudaEventRecord(ev1, s));
+    ACID_CUDA(cudaEventSynchronize(ev1));
+    float ms = 0.f;
+    ACID_CUDA(cudaEventElapsedTime(&ms, ev0, ev1));
+    lg.ms = ms;
+    cudaEventDestroy(ev0);
+    cudaEventDestroy(ev1);
+    *log = lg;
+  }
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_denoise_loop(const acid_model* m, const acid_loop_cfg* cfg, void* latent, const void* text,
+                                         acid_step_log* log, void* workspace, size_t workspace_bytes,
+                                         acid_stream_t stream) {
+  acid_loop_state st;
+  ACID_TRY(acid_loop_begin(m, cfg, text, &st, workspace, workspace_bytes, stream));
+  for (int i = 0; i < cfg->n_steps; ++i)
+    ACID_TRY(acid_denoise_step(m, cfg, &st, latent, log ? log + i : nullptr, workspace, workspace_bytes, stream));
+  return ACID_OK;
+}

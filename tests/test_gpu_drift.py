@@ -1,0 +1,135 @@
+"""GPU parity of the drift signal and cache apply (through the C ABI) against
+the oracle, on the drift micro-benchmark workload ([T, 3072] bf16 pairs,
+T in {4096, 32760, 67320, 118800}, sigma in {1e-3, 1e-2, 1e-1}) and edge
+cases."""
+
+import math
+
+import numpy as np
+import pytest
+
+import acid_synth as S
+import oracle as O
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+DEV = "cuda"
+
+DRIFT_RTOL = 1e-3  # drift values within 1e-3 relative of the oracle
+
+
+@pytest.fixture(scope="module")
+def acid():
+    import __graft_entry__ as g
+
+    g.build()
+    from paper_2607_12358_gb300 import acid as a
+
+    return a
+
+
+def _bf(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(DEV, torch.bfloat16)
+
+
+@pytest.mark.parametrize("T", S.MICRO_T)
+def test_microbench_drift_apply_and_decisions(acid, T):
+    """Full-size micro-benchmark: each sigma's drift value matches the oracle
+    within 1e-3, the fused drift + apply gives the same drift and
+    out = cur + residual to one bf16 rounding, and the dual-threshold decisions
+    on the resulting signal sequence match the oracle's."""
+    r = S.micro_residual(T, seed=5)
+    tr = _bf(r)
+    gpu_s, ref_s = [], []
+    for sigma in S.MICRO_SIGMA:
+        prev, cur = S.micro_pair(T, sigma, seed=5)
+        tp, tc = _bf(prev), _bf(cur)
+        rel, sums = acid.acid_drift_signal(tp, tc)
+        ref = O.rel_l1(prev, cur)
+        num, den = O.drift_sums(prev, cur)
+        assert abs(rel.item() - ref) <= DRIFT_RTOL * ref
+        s = sums.cpu().numpy()
+        assert abs(s[0] - num) <= 1e-4 * num and abs(s[1] - den) <= 1e-4 * den
+        out, rel2, _ = acid.acid_drift_apply(tp, tc, tr)
+        assert abs(rel2.item() - ref) <= DRIFT_RTOL * ref
+        # one rounding of an exact fp32 sum: at most half a bf16 ulp from the rounded fp64 sum
+        ref_out = S.round_to_bf16((cur.astype(np.float64) + r).astype(np.float32))
+        got = out.float().cpu().numpy()
+        ulp = np.abs(ref_out) * 2.0 ** -7 + 1e-30
+        assert np.all(np.abs(got - ref_out) <= ulp)
+        assert np.mean(got == ref_out) > 0.999
+        gpu_s.append(rel.item())
+        ref_s.append(ref)
+        del tp, tc, out
+    # decisions: sigma sweep as a signal sequence under the workload thresholds
+    seq_g = gpu_s * 4
+    seq_r = ref_s * 4
+    d_g = O.controller_decisions(seq_g, 0, 0.05, 0.2, 0.01)
+    d_r = O.controller_decisions(seq_r, 0, 0.05, 0.2, 0.01)
+    assert d_g == d_r
+
+
+def test_drift_identical_is_zero(acid):
+    a = _bf(np.random.default_rng(0).normal(size=12345))
+    rel, sums = acid.acid_drift_signal(a, a)
+    assert rel.item() == 0.0 and sums[0].item() == 0.0
+
+
+def test_drift_zero_denominator(acid):
+    z = torch.zeros(100, device=DEV, dtype=torch.bfloat16)
+    rel, _ = acid.acid_drift_signal(z, z)
+    assert rel.item() == 0.0
+    rel, _ = acid.acid_drift_signal(z, torch.ones_like(z))
+    assert math.isinf(rel.item())
+
+
+@pytest.mark.parametrize("n", [1, 7, 8, 9, 1000, 4097, 3 * 2 ** 20 + 5])
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_drift_ragged_lengths(acid, n, dtype):
+    rng = np.random.default_rng(n)
+    prev = rng.normal(size=n).astype(np.float32)
+    cur = (prev + 0.05 * rng.normal(size=n)).astype(np.float32)
+    if dtype == "bf16":
+        prev, cur = S.round_to_bf16(prev), S.round_to_bf16(cur)
+        tp, tc = _bf(prev), _bf(cur)
+    else:
+        tp, tc = torch.from_numpy(prev).to(DEV), torch.from_numpy(cur).to(DEV)
+    rel, _ = acid.acid_drift_signal(tp, tc)
+    ref = O.rel_l1(prev, cur)
+    assert abs(rel.item() - ref) <= DRIFT_RTOL * ref
+    out = acid.acid_cache_apply(tp, tc)
+    ref_out = (prev.astype(np.float64) + cur).astype(np.float32)
+    if dtype == "bf16":
+        ref_out = S.round_to_bf16(ref_out)
+    np.testing.assert_array_equal(out.float().cpu().numpy(), ref_out)
+
+
+def test_drift_host_output_pointer(acid):
+    """A host output pointer makes the call synchronous and fills host memory."""
+    import ctypes
+    from paper_2607_12358_gb300 import _capi as A
+
+    prev, cur = S.micro_pair(64, 1e-1, seed=9)
+    tp, tc = _bf(prev), _bf(cur)
+    out = ctypes.c_double(-1.0)
+    sums = (ctypes.c_double * 2)()
+    ws = torch.empty(acid.drift_workspace_size(tp.numel()), dtype=torch.uint8, device=DEV)
+    A.check(A.load().acid_drift_signal(tp.data_ptr(), tc.data_ptr(), tp.numel(), A.ACID_BF16, ctypes.addressof(out),
+                                       ctypes.addressof(sums), ws.data_ptr(), ws.numel(),
+                                       torch.cuda.current_stream().cuda_stream))
+    ref = O.rel_l1(prev, cur)
+    assert abs(out.value - ref) <= DRIFT_RTOL * ref
+    assert sums[1] == pytest.approx(O.drift_sums(prev, cur)[1], rel=1e-5)
+
+
+def test_drift_empty_input(acid):
+    e = torch.empty(0, device=DEV, dtype=torch.bfloat16)
+    rel, sums = acid.acid_drift_signal(e, e)
+    assert rel.item() == 0.0
+
+
+def test_drift_rejects_small_workspace(acid):
+    from paper_2607_12358_gb300._capi import AcidError
+    a = torch.zeros(64, device=DEV, dtype=torch.bfloat16)
+    with pytest.raises(AcidError):
+        acid.acid_drift_signal(a, a, workspace=torch.empty(16, dtype=torch.uint8, device=DEV))

@@ -1,0 +1,159 @@
+"""GPU parity of the kernel-level entry points (through the C ABI) against
+the CPU oracle's definitions of the same operations."""
+
+import numpy as np
+import pytest
+
+import acid_synth as S
+import oracle as O
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def acid():
+    import __graft_entry__ as g
+
+    g.build()
+    from paper_2607_12358_gb300 import acid as a
+
+    return a
+
+
+DEV = "cuda"
+
+
+def _bf(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(DEV, torch.bfloat16)
+
+
+def _f32(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(DEV)
+
+
+def _rel_l2(got, ref):
+    return float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30))
+
+
+# ---------------------------------------------------------------------------
+# Linear layers (tcgen05 GEMM, bf16 in / fp32 accumulate)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("M,K,N", [(128, 64, 64), (200, 128, 256), (333, 192, 128), (1000, 1536, 768),
+                                   (64, 4096, 3072), (257, 64, 96)])
+def test_linear_bf16_bias(acid, M, K, N):
+    rng = np.random.default_rng(M + K + N)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.05 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    out = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), out_fp32=True)
+    ref = O.linear(a, w, b)
+    got = out.cpu().numpy()
+    # fp32 accumulation of bf16 products: error ~ sqrt(K) * 2^-24 * |terms|
+    assert np.abs(got - ref).max() <= 1e-4 * (1 + np.abs(ref).max()), np.abs(got - ref).max()
+
+
+@pytest.mark.parametrize("epi", ["bias", "gelu", "gated_res", "res"])
+def test_linear_bf16_epilogues(acid, epi):
+    M, K, N = 300, 256, 512
+    rng = np.random.default_rng(7)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.1 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    g = rng.normal(size=N).astype(np.float32)
+    r = S.round_to_bf16(rng.normal(size=(M, N)).astype(np.float32))
+    res = _bf(r)
+    out = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), epilogue=epi, gate=_f32(g),
+                                   residual=res if epi in ("gated_res", "res") else None,
+                                   out=res if epi in ("gated_res", "res") else None)
+    acc = O.linear(a, w, b)
+    ref = {"bias": acc, "gelu": O.gelu_tanh(acc), "gated_res": r + g * acc, "res": r + acc}[epi]
+    got = out.float().cpu().numpy()
+    # bf16 output: one rounding (2^-9 relative) plus the tanh approximation for GELU
+    assert np.abs(got - ref).max() <= 2 ** -8 * (np.abs(ref).max() + 1), np.abs(got - ref).max()
+    assert _rel_l2(got, ref) <= 4e-3
+
+
+def test_linear_fp32(acid):
+    M, K, N = 77, 96, 130
+    rng = np.random.default_rng(8)
+    a, w, b = rng.normal(size=(M, K)), rng.normal(size=(N, K)), rng.normal(size=N)
+    out = acid.acid_linear_forward(_f32(a), _f32(w), _f32(b), epilogue="gelu")
+    ref = O.gelu_tanh(O.linear(a.astype(np.float32), w.astype(np.float32), b.astype(np.float32)))
+    assert _rel_l2(out.cpu().numpy(), ref) <= 1e-5
+
+
+def test_linear_rejects_bad_shapes(acid):
+    from paper_2607_12358_gb300._capi import AcidError
+    a = torch.zeros(10, 64, device=DEV, dtype=torch.bfloat16)
+    w = torch.zeros(40, 64, device=DEV, dtype=torch.bfloat16)  # N % 32 != 0
+    with pytest.raises(AcidError):
+        acid.acid_linear_forward(a, w)
+
+
+# ---------------------------------------------------------------------------
+# Attention (tcgen05 flash attention)
+# ---------------------------------------------------------------------------
+
+def _attn_case(nq, nk, H, D, seed, qscale=1.0):
+    rng = np.random.default_rng(seed)
+    q = S.round_to_bf16((qscale * rng.normal(size=(nq, H * D))).astype(np.float32))
+    k = S.round_to_bf16(rng.normal(size=(nk, H * D)).astype(np.float32))
+    v = S.round_to_bf16(rng.normal(size=(nk, H * D)).astype(np.float32))
+    ref = O.attention(q.reshape(nq, H, D), k.reshape(nk, H, D), v.reshape(nk, H, D)).reshape(nq, H * D)
+    return q, k, v, ref
+
+
+@pytest.mark.parametrize("nq,nk,H,D,qscale", [(128, 128, 1, 128, 1.0), (300, 300, 2, 128, 1.0),
+                                              (300, 257, 2, 64, 2.0), (1000, 512, 3, 128, 3.0),
+                                              (129, 1000, 2, 64, 4.0), (2048, 2048, 2, 128, 1.0)])
+def test_attention_bf16(acid, nq, nk, H, D, qscale):
+    q, k, v, ref = _attn_case(nq, nk, H, D, nq + nk, qscale)
+    out = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), H)
+    got = out.float().cpu().numpy()
+    assert _rel_l2(got, ref) <= 1e-2, _rel_l2(got, ref)
+    assert np.abs(got - ref).max() <= 5e-2
+
+
+def test_attention_one_key_returns_value(acid):
+    q, k, v, ref = _attn_case(200, 1, 2, 128, 3)
+    got = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), 2).float().cpu().numpy()
+    np.testing.assert_array_equal(got, np.broadcast_to(v, got.shape))
+
+
+def test_attention_peaky_rescaling(acid):
+    """Logits spanning far more than 2^8 across key tiles exercise the
+    deferred rescaling of the output accumulator."""
+    q, k, v, ref = _attn_case(256, 1024, 1, 128, 5, qscale=1.0)
+    k = k.copy()
+    k[900:] *= 12.0  # late keys dominate: the running max jumps in the last tiles
+    k = S.round_to_bf16(k)
+    ref = O.attention(q.reshape(256, 1, 128), k.reshape(1024, 1, 128), v.reshape(1024, 1, 128)).reshape(256, 128)
+    got = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), 1).float().cpu().numpy()
+    assert _rel_l2(got, ref) <= 1e-2
+
+
+def test_attention_fp32(acid):
+    rng = np.random.default_rng(11)
+    q, k, v = (rng.normal(size=(70, 128)) for _ in range(3))
+    ref = O.attention(q.reshape(70, 2, 64), k.reshape(70, 2, 64), v.reshape(70, 2, 64)).reshape(70, 128)
+    got = acid.acid_attention_forward(_f32(q), _f32(k), _f32(v), 2).cpu().numpy()
+    assert _rel_l2(got, ref) <= 1e-5
+
+
+# ---------------------------------------------------------------------------
+# adaLN LayerNorm
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("d", [256, 1536, 1920, 3072])
+def test_layernorm_mod(acid, d):
+    rng = np.random.default_rng(d)
+    x = S.round_to_bf16((2.0 + 3.0 * rng.normal(size=(333, d))).astype(np.float32))
+    sh, sc = rng.normal(size=d).astype(np.float32), rng.normal(size=d).astype(np.float32)
+    ref = O.modulate(O.layer_norm(x), sh, sc)
+    got = acid.acid_layernorm_mod(_bf(x), _f32(sh), _f32(sc), out_dtype=torch.float32).cpu().numpy()
+    assert np.abs(got - ref).max() <= 1e-4 * (1 + np.abs(ref).max())
+    got16 = acid.acid_layernorm_mod(_bf(x), _f32(sh), _f32(sc)).float().cpu().numpy()
+    assert np.abs(got16 - ref).max() <= 2 ** -8 * (1 + np.abs(ref).max())

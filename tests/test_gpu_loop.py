@@ -1,0 +1,149 @@
+"""GPU parity of the step loop (acid_denoise_loop / acid_denoise_step through
+the C ABI) against the oracle's Algorithm 1 loop.
+
+* fp32 toy workload (2 blocks, d=256, 10 Euler steps, TeaCache signal,
+  tau_low=0.05, tau_high=0.2): whole loop against the oracle; decisions
+  identical except at ambiguous steps (accumulated drift within 1e-3
+  relative of the threshold, or |s_t - s_prev| within 1e-3 of delta), where
+  the oracle is re-run with the GPU's decision forced.
+* EasyCache variant of the toy loop, same protocol.
+* bf16 small Wan-shaped loop: teacher-forced signal check (the oracle
+  recomputes s_t from the GPU's own latents, within 1e-3) and controller
+  replay (the oracle controller fed the GPU's signals takes the same
+  decisions).
+"""
+
+import math
+
+import numpy as np
+import pytest
+
+import acid_synth as S
+import oracle as O
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def acid():
+    import __graft_entry__ as g
+
+    g.build()
+    from paper_2607_12358_gb300 import acid as a
+
+    return a
+
+
+def _ambiguous(rec_sigma, rec_tau, ds, delta):
+    if rec_tau != rec_tau:  # warmup
+        return False
+    if abs(rec_sigma - rec_tau) <= 1e-3 * max(abs(rec_tau), 1e-12):
+        return True
+    return ds == ds and abs(ds - delta) <= 1e-3 * max(abs(delta), 1e-6)
+
+
+def _compare_loop(acid, cfg, w, lat, text=None, **kw):
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg, **kw)
+    tl = torch.from_numpy(lat).to(DEV)
+    tt = None if text is None else torch.from_numpy(text).to(DEV, model.wdtype)
+    logs = acid.acid_denoise_loop(model, c, tl, tt)
+    acid.check_device_error()
+    gpu_dec = [bool(l["computed"]) for l in logs]
+    okw = {k: v for k, v in kw.items() if k in ("tau_low", "tau_high", "delta", "method", "n_steps")}
+    ref = O.denoise_loop(cfg, w, lat, text, **okw)
+    forced = [None] * len(gpu_dec)
+    for i in range(len(gpu_dec)):
+        rec = ref.records[i]
+        if rec.computed != gpu_dec[i]:
+            assert _ambiguous(rec.sigma, rec.tau, rec.dsignal, c.delta), (i, rec, logs[i])
+            forced[i] = gpu_dec[i]
+            ref = O.denoise_loop(cfg, w, lat, text, forced=forced, **okw)
+    assert [r.computed for r in ref.records] == gpu_dec
+    for l, r in zip(logs, ref.records):
+        if not r.warmup:
+            assert abs(l["signal"] - r.signal) <= 1e-3 * abs(r.signal) + 1e-12, (l, r)
+    return tl.cpu().numpy(), ref, logs
+
+
+def test_toy_loop_teacache(acid):
+    cfg = S.get_config("toy")
+    w = S.model_weights(cfg, 0)
+    lat = S.latent(cfg, 0)
+    got, ref, logs = _compare_loop(acid, cfg, w, lat)
+    err = np.abs(got - ref.latent).max() / np.abs(ref.latent).max()
+    assert err <= 1e-4, err
+    assert 0 < sum(ref.computed) < cfg.steps  # the workload exercises both branches
+
+
+@pytest.mark.parametrize("tau", [(-1.0, -1.0), (1e9, 1e9), (0.05, 0.05)])
+def test_toy_loop_threshold_extremes(acid, tau):
+    cfg = S.get_config("toy", steps=6)
+    w = S.model_weights(cfg, 1)
+    lat = S.latent(cfg, 1)
+    got, ref, _ = _compare_loop(acid, cfg, w, lat, tau_low=tau[0], tau_high=tau[1])
+    assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+
+
+def test_toy_loop_easycache(acid):
+    cfg = S.get_config("toy", method="easycache", tau_low=0.02, tau_high=0.04, steps=10)
+    w = S.model_weights(cfg, 2)
+    lat = S.latent(cfg, 2)
+    got, ref, _ = _compare_loop(acid, cfg, w, lat, method="easycache")
+    assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+
+
+def test_toy_loop_forced_decisions(acid):
+    cfg = S.get_config("toy", steps=6)
+    w = S.model_weights(cfg, 3)
+    lat = S.latent(cfg, 3)
+    forced = [None, False, True, False, None, True]
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg, forced=forced)
+    tl = torch.from_numpy(lat).to(DEV)
+    logs = acid.acid_denoise_loop(model, c, tl)
+    ref = O.denoise_loop(cfg, w, lat, None, forced=forced)
+    assert [bool(l["computed"]) for l in logs] == ref.computed
+    assert np.abs(tl.cpu().numpy() - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+
+
+@pytest.mark.parametrize("kind", ["wan", "cog", "hv"])
+def test_bf16_loop_teacher_forced_signal_and_replay(acid, kind):
+    over = dict(d=256, heads=2, ffn=512, latent_f=3, latent_h=16, latent_w=22, steps=8)
+    if kind == "wan":
+        cfg = S.get_config("wan", n_blocks=2, n_text=40, d_text=256, **over)
+    elif kind == "cog":
+        over["heads"] = 4
+        cfg = S.get_config("cog", n_blocks=2, n_text=30, d_text=256, **over)
+    else:
+        cfg = S.get_config("hv", n_blocks=1, n_single=1, n_text=30, d_text=256, **over)
+    w = S.model_weights(cfg, 4)
+    lat = S.latent(cfg, 4)
+    text = S.text(cfg, 4)
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg)
+    tt = torch.from_numpy(text).to(DEV, torch.bfloat16)
+    loop = acid.Loop(model, c, tt, DEV)
+    tl = torch.from_numpy(lat).to(DEV)
+    xs, logs = [], []
+    for i in range(cfg.steps):
+        xs.append(tl.cpu().numpy().astype(np.float64))
+        logs.append(acid.log_to_dict(loop.step(tl)))
+    acid.check_device_error()
+    sig = O.sigmas(cfg.steps)
+    W = cfg.warmup
+    # teacher-forced signal
+    if cfg.method == "teacache":
+        temni = [O.block0_temni(cfg, w, O.step_inputs(cfg, w, x, 1000 * sig[i], with_blocks=False).h_in,
+                                O.time_embedding(1000 * sig[i], w, cfg.time_freq_dim)) for i, x in enumerate(xs)]
+        for i in range(W, cfg.steps):
+            ref = O.rel_l1(temni[i - 1], temni[i])
+            assert abs(logs[i]["signal"] - ref) <= 1e-3 * ref, (i, logs[i]["signal"], ref)
+    # controller replay
+    gpu_s = [l["signal"] if i >= W else 0.0 for i, l in enumerate(logs)]
+    dec = O.controller_decisions(gpu_s, W, cfg.tau_low, cfg.tau_high, cfg.delta)
+    assert dec == [bool(l["computed"]) for l in logs]
+    assert all(math.isfinite(l["signal"]) for l in logs[W:])
+    assert np.isfinite(tl.cpu().numpy()).all()
