@@ -11,7 +11,7 @@ namespace acid {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kDriftMaxBlocks = 152 * 8;  // one wave of 8 CTAs per SM on GB300
+constexpr int kDriftMaxBlocks = 152 * 4;  // one wave of 4 CTAs per SM on GB300
 
 __device__ __forceinline__ double warp_sum_d(double v) {
 #pragma unroll
@@ -43,47 +43,70 @@ template <> struct Vec<float> {
 
 // One pass over prev/cur: per-thread fp32 sums of |cur - prev| and |prev|,
 // fp64 across the CTA, one partial per CTA.  kApply also writes
-// out = cur + resid in the same pass.
+// out = cur + resid in the same pass.  Loads are raw 16-byte vectors, U of
+// them in flight per tensor and thread, unpacked after all have been issued.
+template <typename T>
+__device__ __forceinline__ void unpack16(const uint4& u, float* v);
+template <>
+__device__ __forceinline__ void unpack16<__nv_bfloat16>(const uint4& u, float* v) {
+  v[0] = bf16_lo(u.x); v[1] = bf16_hi(u.x); v[2] = bf16_lo(u.y); v[3] = bf16_hi(u.y);
+  v[4] = bf16_lo(u.z); v[5] = bf16_hi(u.z); v[6] = bf16_lo(u.w); v[7] = bf16_hi(u.w);
+}
+template <>
+__device__ __forceinline__ void unpack16<float>(const uint4& u, float* v) {
+  v[0] = __uint_as_float(u.x); v[1] = __uint_as_float(u.y); v[2] = __uint_as_float(u.z); v[3] = __uint_as_float(u.w);
+}
+
 template <typename T, bool kApply>
-__global__ void __launch_bounds__(kThreads) drift_partials_kernel(const T* __restrict__ prev,
-                                                                  const T* __restrict__ cur,
-                                                                  const T* __restrict__ resid, T* out,
-                                                                  int64_t n, double2* __restrict__ partials) {
+__global__ void __launch_bounds__(kThreads, 4) drift_partials_kernel(const T* __restrict__ prev,
+                                                                     const T* __restrict__ cur,
+                                                                     const T* __restrict__ resid, T* out,
+                                                                     int64_t n, double2* __restrict__ partials) {
   constexpr int V = Vec<T>::N;
-  constexpr int U = 4;  // vectors in flight per thread and tensor
+  constexpr int U = kApply ? 2 : 4;  // 16-byte vectors in flight per thread and tensor
   const int64_t nvec = n / V;
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  float num = 0.f, den = 0.f;
+  const uint4* p4 = reinterpret_cast<const uint4*>(prev);
+  const uint4* c4 = reinterpret_cast<const uint4*>(cur);
+  const uint4* r4 = reinterpret_cast<const uint4*>(resid);
+  float num0 = 0.f, num1 = 0.f, den0 = 0.f, den1 = 0.f;
   for (int64_t base = tid; base < nvec; base += U * stride) {
-    float p[U][V], c[U][V], r[U][V];
+    uint4 pr[U], cr[U], rr[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int64_t i = base + u * stride;
       if (i < nvec) {
-        Vec<T>::ld(prev + i * V, p[u]);
-        Vec<T>::ld(cur + i * V, c[u]);
-        if (kApply) Vec<T>::ld(resid + i * V, r[u]);
+        pr[u] = __ldcs(p4 + i);
+        cr[u] = __ldcs(c4 + i);
+        if (kApply) rr[u] = __ldcs(r4 + i);
       }
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int64_t i = base + u * stride;
       if (i < nvec) {
+        float p[V], c[V];
+        unpack16<T>(pr[u], p);
+        unpack16<T>(cr[u], c);
 #pragma unroll
-        for (int j = 0; j < V; ++j) {
-          num += fabsf(c[u][j] - p[u][j]);
-          den += fabsf(p[u][j]);
+        for (int j = 0; j < V; j += 2) {
+          num0 += fabsf(c[j] - p[j]);
+          num1 += fabsf(c[j + 1] - p[j + 1]);
+          den0 += fabsf(p[j]);
+          den1 += fabsf(p[j + 1]);
         }
         if (kApply) {
-          float o[V];
+          float r[V];
+          unpack16<T>(rr[u], r);
 #pragma unroll
-          for (int j = 0; j < V; ++j) o[j] = c[u][j] + r[u][j];
-          Vec<T>::st(out + i * V, o);
+          for (int j = 0; j < V; ++j) r[j] += c[j];
+          Vec<T>::st(out + i * V, r);
         }
       }
     }
   }
+  float num = num0 + num1, den = den0 + den1;
   for (int64_t i = nvec * V + tid; i < n; i += stride) {  // ragged tail
     const float pv = io<T>::ld(prev + i), cv = io<T>::ld(cur + i);
     num += fabsf(cv - pv);

@@ -109,10 +109,16 @@ __device__ __forceinline__ void epi_pair(const EpiDev& e, int64_t grow, int col,
 __host__ __device__ __forceinline__ bool epi_reads_res(int kind) { return kind == EPI_GATED_RES || kind == EPI_RES; }
 
 // ===========================================================================
-// tcgen05 GEMM (bf16 in, fp32 accumulate)
+// tcgen05 GEMM (bf16 in, fp32 accumulate), persistent
+//
+// One CTA per SM walks output tiles (N fastest, so the CTAs running together
+// share A row blocks in L2 and the weight tiles stay L2-resident).  The TMEM
+// accumulator is double-buffered (2 x BN columns): the MMA warp fills buffer
+// b for tile i+1 while eight epilogue warps drain buffer b^1 of tile i.
 // ===========================================================================
 constexpr int BM = 128, BK = 64;
-constexpr int kGemmThreads = 192;
+constexpr int kEpiWarps = 8;
+constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
 
 template <int BN>
 struct TcCfg {
@@ -121,6 +127,7 @@ struct TcCfg {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
 struct GemmDims {
@@ -130,6 +137,41 @@ struct GemmDims {
   int64_t ldo;
   int out_fp32;
 };
+
+template <int BN>
+__device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, int64_t row, int col0,
+                                               const uint32_t* r) {
+  const int64_t grow = row + e.row_base;
+  float v[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+  float rv[32];
+  if (epi_reads_res(e.kind)) {
+    if (g.out_fp32) {
+      const float* rp = static_cast<const float*>(e.res) + row * e.ldr + col0;
+#pragma unroll
+      for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
+    } else {
+      const __nv_bfloat16* rp = static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col0;
+#pragma unroll
+      for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) rv[j] = 0.f;
+  }
+#pragma unroll
+  for (int j = 0; j < 32; j += 2) epi_pair<true>(e, grow, col0 + j, v[j], v[j + 1], rv[j], rv[j + 1]);
+  if (g.out_fp32) {
+    float* op = static_cast<float*>(g.out) + row * g.ldo + col0;
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
+  } else {
+    __nv_bfloat16* op = static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col0;
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
+  }
+}
 
 template <int BN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
@@ -142,12 +184,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
   uint64_t* empty = full + C::STAGES;
-  uint64_t* accum = empty + C::STAGES;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  uint64_t* acc_full = empty + C::STAGES;  // [2]
+  uint64_t* acc_empty = acc_full + 2;      // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_tile = blockIdx.x, m_tile = blockIdx.y;
   const int num_kb = (g.K + BK - 1) / BK;
+  const int num_n = (g.N + BN - 1) / BN;
+  const int num_tiles = (int)((g.M + BM - 1) / BM) * num_n;
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
@@ -156,95 +200,89 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(accum, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 32 * kEpiWarps);
+    }
     mbar_fence_init();
   }
-  if (warp == 1) tmem_alloc(tmem_slot, BN);
+  if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    if (lane == 0) {  // TMA producer
-      for (int kb = 0; kb < num_kb; ++kb) {
-        const int s = kb % C::STAGES, round = kb / C::STAGES;
-        if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1)) break;
-        mbar_expect_tx(&full[s], C::STAGE_BYTES);
-        tma_load_2d(sA + s * C::A_BYTES, &tmA, &full[s], kb * BK, m_tile * BM);
-        tma_load_2d(sB + s * C::B_BYTES, &tmB, &full[s], kb * BK, n_tile * BN);
+    if (lane == 0) {  // TMA producer: one continuous stage ring across tiles
+      int it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
+        const int m_tile = tile / num_n, n_tile = tile % num_n;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % C::STAGES, round = it / C::STAGES;
+          if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1)) { ok = false; break; }
+          mbar_expect_tx(&full[s], C::STAGE_BYTES);
+          tma_load_2d(sA + s * C::A_BYTES, &tmA, &full[s], kb * BK, m_tile * BM);
+          tma_load_2d(sB + s * C::B_BYTES, &tmB, &full[s], kb * BK, n_tile * BN);
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {  // MMA issuer
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
+      int it = 0, local = 0;
       bool ok = true;
-      for (int kb = 0; kb < num_kb && ok; ++kb) {
-        const int s = kb % C::STAGES, round = kb / C::STAGES;
-        if (!mbar_wait(&full[s], round & 1)) { ok = false; break; }
+      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++local) {
+        const int b = local & 1, use = local >> 1;
+        if (use > 0 && !mbar_wait(&acc_empty[b], (use - 1) & 1)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
-        const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+        const uint32_t d = tmem + b * BN;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % C::STAGES, round = it / C::STAGES;
+          if (!mbar_wait(&full[s], round & 1)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-          const uint64_t ad = smem_desc_sw128(a0 + k * 32, 16, 1024);
-          const uint64_t bd = smem_desc_sw128(b0 + k * 32, 16, 1024);
-          mma_bf16_ss(tmem, ad, bd, idesc, (kb | k) != 0);
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t ad = smem_desc_sw128(a0 + k * 32, 16, 1024);
+            const uint64_t bd = smem_desc_sw128(b0 + k * 32, 16, 1024);
+            mma_bf16_ss(d, ad, bd, idesc, (kb | k) != 0);
+          }
+          mma_commit(&empty[s]);
         }
-        mma_commit(&empty[s]);
+        if (ok) mma_commit(&acc_full[b]);
       }
-      if (ok) mma_commit(accum);
     }
-  } else {  // epilogue: warps 2..5 -> TMEM lane quarters 2, 3, 0, 1
-    const int q = warp & 3;
-    const bool ok = mbar_wait(accum, 0);
-    tc_fence_after();
-    const int64_t row = (int64_t)m_tile * BM + q * 32 + lane;
-    const int64_t grow = row + e.row_base;
-    const bool row_ok = ok && row < g.M;
+  } else {  // epilogue: warps 2..9; lane quarter = warp % 4, column half = (warp - 2) / 4
+    const int q = warp & 3, half = (warp - 2) >> 2;
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    int local = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+      const int b = local & 1, use = local >> 1;
+      const int m_tile = tile / num_n, n_tile = tile % num_n;
+      const bool ok = mbar_wait(&acc_full[b], use & 1);
+      tc_fence_after();
+      const int64_t row = (int64_t)m_tile * BM + q * 32 + lane;
+      const bool row_ok = ok && row < g.M;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + c, r);
-      tmem_wait_ld();
-      const int col0 = n_tile * BN + c;
-      if (!row_ok || col0 >= g.N) continue;
-      float v[32];
-#pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-      float rv[32];
-      if (epi_reads_res(e.kind)) {
-        if (g.out_fp32) {
-          const float* rp = static_cast<const float*>(e.res) + row * e.ldr + col0;
-#pragma unroll
-          for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
-        } else {
-          const __nv_bfloat16* rp = static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col0;
-#pragma unroll
-          for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
-        }
-      } else {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) rv[j] = 0.f;
+      for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+        uint32_t r[32];
+        tmem_ld32(tmem + lane_base + b * BN + c, r);
+        tmem_wait_ld();
+        const int col0 = n_tile * BN + c;
+        if (row_ok && col0 < g.N) epilogue_chunk<BN>(g, e, row, col0, r);
       }
-#pragma unroll
-      for (int j = 0; j < 32; j += 2) epi_pair<true>(e, grow, col0 + j, v[j], v[j + 1], rv[j], rv[j + 1]);
-      if (g.out_fp32) {
-        float* op = static_cast<float*>(g.out) + row * g.ldo + col0;
-#pragma unroll
-        for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
-      } else {
-        __nv_bfloat16* op = static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col0;
-#pragma unroll
-        for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
-      }
+      tc_fence_before();
+      mbar_arrive(&acc_empty[b]);
+      if (!ok) break;
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, BN);
+    tmem_dealloc(tmem, C::TMEM_COLS);
   }
 }
 
@@ -287,6 +325,16 @@ acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int
 
 namespace {
 
+int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  }
+  return n;
+}
+
 template <int BN>
 acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
                       const Epilogue& epi, cudaStream_t s) {
@@ -300,7 +348,8 @@ acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* 
   ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
   ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, BN));
   GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0};
-  dim3 grid((N + BN - 1) / BN, (unsigned)((M + BM - 1) / BM));
+  const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+  const int grid = (int)std::min<int64_t>(tiles, num_sms());
   ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
   gemm_tc_kernel<BN><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
   ACID_CHECK_LAUNCH();
