@@ -4,18 +4,21 @@
 // operands.
 //
 // bf16 path: a flash-attention kernel on tcgen05 tensor cores.  One CTA owns
-// 128 query rows of one head:
-//   warp 0      TMA producer: Q once, then K_j / V_j tiles of 128 keys into a
-//               2-deep ring (128-byte swizzle);
-//   warp 1      MMA issuer: S_j = Q K_j^T into one of two TMEM S buffers,
-//               then O += P_{j-1} V_{j-1} into the TMEM O accumulator, so the
-//               tensor core computes S_{j+1} while softmax works on S_j;
-//   warps 4-7   softmax: one thread per query row reads its S row from TMEM,
-//               keeps the running max and sum, writes P (bf16) to shared
-//               memory in the swizzled K-major layout the MMA reads, and
-//               rescales O in TMEM only when the running max grows by more
-//               than 2^8 (the final division by the sum makes the result
-//               independent of when rescaling happens).
+// two 128-row query tiles (a, b) of one head and streams 128-key K/V tiles
+// that both query tiles share:
+//   warp 0      TMA producer: Q_a, Q_b once, then K_j and V_j into 2-deep rings
+//               (128-byte swizzle);
+//   warp 1      MMA issuer, in the order S_a(0) S_b(0) | PV_a(j) S_a(j+1)
+//               PV_b(j) S_b(j+1) | ... so that the tensor core works on one
+//               query tile while the softmax of the other runs;
+//               S_t = Q_t K_j^T lands in TMEM, P_t is written back over S_t
+//               (bf16, two per column) and O_t += P_t V_j reads P_t from TMEM
+//               and V_j from shared memory;
+//   warps 2-5   softmax of tile a, warps 6-9 softmax of tile b: one thread
+//               per query row keeps the running max and sum, and rescales O_t
+//               in TMEM only when the running max grows by more than 2^8 (the
+//               final division by the sum makes the result independent of
+//               when rescaling happens).
 // fp32 path: one warp per query row, exact expf, for the fp32 mode.
 #include <cudaTypedefs.h>
 #include <math.h>
@@ -29,9 +32,10 @@ acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int
 
 namespace {
 
-constexpr int kBQ = 128;   // query rows per CTA
-constexpr int kBKV = 128;  // keys per tile
-constexpr int kAttnThreads = 256;
+constexpr int kTileQ = 128;  // query rows per tile (two tiles per CTA)
+constexpr int kBQ = 2 * kTileQ;
+constexpr int kBKV = 128;  // keys per K/V tile
+constexpr int kAttnThreads = 320;
 constexpr float kRescaleLog2 = 8.0f;
 
 struct AttnDev {
@@ -47,16 +51,16 @@ template <int D>
 struct AttnCfg {
   static constexpr int CH = D / 64;                 // 64-column chunks per row
   static constexpr int CHUNK_BYTES = 128 * 128;     // 128 rows x 128 bytes
-  static constexpr int Q_BYTES = CH * CHUNK_BYTES;  // also K / V tile bytes
-  static constexpr int P_BYTES = 2 * CHUNK_BYTES;   // 128 x 128 bf16
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + Q_BYTES;
-  static constexpr int OFF_V = OFF_K + 2 * Q_BYTES;
-  static constexpr int OFF_P = OFF_V + 2 * Q_BYTES;
-  static constexpr int OFF_BAR = OFF_P + P_BYTES;
+  static constexpr int T_BYTES = CH * CHUNK_BYTES;  // one 128-row tile of Q, K or V
+  static constexpr int OFF_Q = 0;                   // Q_a, Q_b
+  static constexpr int OFF_K = OFF_Q + 2 * T_BYTES;
+  static constexpr int OFF_V = OFF_K + 2 * T_BYTES;
+  static constexpr int OFF_BAR = OFF_V + 2 * T_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  static constexpr uint32_t TMEM_COLS = 512;  // S0 [0,128), S1 [128,256), O [256, 256+D)
-  static constexpr uint32_t O_COL = 256;
+  // TMEM columns: S_a [0,128), S_b [128,256) (P_t over the first 64 columns of
+  // S_t), O_a [256, 256+D), O_b [384, 384+D)
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t S_COL = 0, O_COL = 256;
 };
 
 template <int D>
@@ -69,17 +73,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   uint8_t* sQ = smem + C::OFF_Q;
   uint8_t* sK = smem + C::OFF_K;
   uint8_t* sV = smem + C::OFF_V;
-  uint8_t* sP = smem + C::OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;   // [2]
-  uint64_t* k_empty = bars + 3;  // [2]
-  uint64_t* v_full = bars + 5;   // [2]
-  uint64_t* v_empty = bars + 7;  // [2]
-  uint64_t* s_full = bars + 9;   // [2]
-  uint64_t* s_free = bars + 11;  // [2]
-  uint64_t* p_full = bars + 13;
-  uint64_t* pv_done = bars + 14;
+  uint64_t* k_full = bars + 1;    // [2]
+  uint64_t* k_empty = bars + 3;   // [2]
+  uint64_t* v_full = bars + 5;    // [2]
+  uint64_t* v_empty = bars + 7;   // [2]
+  uint64_t* s_full = bars + 9;    // [2] per query tile
+  uint64_t* p_full = bars + 11;   // [2] per query tile
+  uint64_t* pv_done = bars + 13;  // [2] per query tile
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -97,10 +99,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(&v_full[i], 1);
       mbar_init(&v_empty[i], 1);
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 128);
+      mbar_init(&p_full[i], 128);
+      mbar_init(&pv_done[i], 1);
     }
-    mbar_init(p_full, 128);
-    mbar_init(pv_done, 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -111,20 +112,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------------------------------- TMA producer
-      mbar_expect_tx(q_full, C::Q_BYTES);
-      for (int c = 0; c < C::CH; ++c)
-        tma_load_2d(sQ + c * C::CHUNK_BYTES, &tmQ, q_full, a.q_col + h * D + c * 64, qt * kBQ);
+      mbar_expect_tx(q_full, 2 * C::T_BYTES);
+      for (int t = 0; t < 2; ++t)
+        for (int c = 0; c < C::CH; ++c)
+          tma_load_2d(sQ + t * C::T_BYTES + c * C::CHUNK_BYTES, &tmQ, q_full, a.q_col + h * D + c * 64,
+                      qt * kBQ + t * kTileQ);
       for (int j = 0; j < nkv; ++j) {
         const int st = j & 1, round = j >> 1;
         if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) break;
-        mbar_expect_tx(&k_full[st], C::Q_BYTES);
+        mbar_expect_tx(&k_full[st], C::T_BYTES);
         for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sK + st * C::Q_BYTES + c * C::CHUNK_BYTES, &tmK, &k_full[st], a.k_col + h * D + c * 64,
+          tma_load_2d(sK + st * C::T_BYTES + c * C::CHUNK_BYTES, &tmK, &k_full[st], a.k_col + h * D + c * 64,
                       j * kBKV);
         if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) break;
-        mbar_expect_tx(&v_full[st], C::Q_BYTES);
+        mbar_expect_tx(&v_full[st], C::T_BYTES);
         for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sV + st * C::Q_BYTES + c * C::CHUNK_BYTES, &tmV, &v_full[st], a.v_col + h * D + c * 64,
+          tma_load_2d(sV + st * C::T_BYTES + c * C::CHUNK_BYTES, &tmV, &v_full[st], a.v_col + h * D + c * 64,
                       j * kBKV);
       }
     }
@@ -132,58 +135,67 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (lane == 0) {  // ---------------------------------------- MMA issuer
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, kBKV, false, false);
       constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
-      bool ok = mbar_wait(q_full, 0);
-      const uint32_t q0 = smem_u32(sQ), p0 = smem_u32(sP);
-      for (int j = 0; ok && j <= nkv; ++j) {
-        if (j < nkv) {
-          const int st = j & 1;
-          if (!mbar_wait(&k_full[st], (j >> 1) & 1)) { ok = false; break; }
-          if (j >= 2 && !mbar_wait(&s_free[st], ((j >> 1) - 1) & 1)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t k0 = smem_u32(sK + st * C::Q_BYTES);
+      const uint32_t q0 = smem_u32(sQ);
+      // S_t(j) = Q_t K_j^T into the S region of tile t
+      auto issue_s = [&](int t, int j) {
+        const uint32_t k0 = smem_u32(sK + (j & 1) * C::T_BYTES);
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
-            mma_bf16_ss(tmem + st * kBKV, smem_desc_sw128(q0 + off, 16, 1024), smem_desc_sw128(k0 + off, 16, 1024),
-                        idesc_s, kk != 0);
-          }
-          mma_commit(&k_empty[st]);
-          mma_commit(&s_full[st]);
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
+          mma_bf16_ss(tmem + C::S_COL + t * kBKV, smem_desc_sw128(q0 + t * C::T_BYTES + off, 16, 1024),
+                      smem_desc_sw128(k0 + off, 16, 1024), idesc_s, kk != 0);
         }
-        if (j >= 1) {
-          const int jp = j - 1, st = jp & 1;
-          if (!mbar_wait(p_full, jp & 1)) { ok = false; break; }
-          if (!mbar_wait(&v_full[st], (jp >> 1) & 1)) { ok = false; break; }
+        mma_commit(&s_full[t]);
+      };
+      bool ok = mbar_wait(q_full, 0) && mbar_wait(&k_full[0], 0);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+        mma_commit(&k_empty[0]);
+      }
+      for (int j = 0; ok && j < nkv; ++j) {
+        const int st = j & 1;
+        for (int t = 0; t < 2 && ok; ++t) {
+          if (!mbar_wait(&p_full[t], j & 1)) { ok = false; break; }
+          if (t == 0 && !mbar_wait(&v_full[st], (j >> 1) & 1)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t v0 = smem_u32(sV + st * C::Q_BYTES);
+          // O_t += P_t V_j: P_t (128 x 128 keys) from TMEM, V_j MN-major from shared memory
+          const uint32_t v0 = smem_u32(sV + st * C::T_BYTES);
 #pragma unroll
-          for (int kk = 0; kk < kBKV / 16; ++kk) {
-            const uint32_t poff = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
-            // V is MN-major: 16 key rows of 128 bytes per step; 64-column chunks 16 KB apart
-            mma_bf16_ss(tmem + C::O_COL, smem_desc_sw128(p0 + poff, 16, 1024),
-                        smem_desc_sw128(v0 + kk * 16 * 128, C::CHUNK_BYTES, 1024), idesc_o, (jp | kk) != 0);
+          for (int kk = 0; kk < kBKV / 16; ++kk)
+            mma_bf16_ts(tmem + C::O_COL + t * 128, tmem + C::S_COL + t * kBKV + kk * 8,
+                        smem_desc_sw128(v0 + kk * 16 * 128, C::CHUNK_BYTES, 1024), idesc_o, (j | kk) != 0);
+          mma_commit(&pv_done[t]);
+          if (t == 1) mma_commit(&v_empty[st]);
+          if (j + 1 < nkv) {
+            if (t == 0 && !mbar_wait(&k_full[st ^ 1], ((j + 1) >> 1) & 1)) { ok = false; break; }
+            tc_fence_after();
+            issue_s(t, j + 1);
+            if (t == 1) mma_commit(&k_empty[st ^ 1]);
           }
-          mma_commit(&v_empty[st]);
-          mma_commit(pv_done);
         }
       }
     }
-  } else if (warp >= 4) {  // ---------------------------------------- softmax
+  } else {  // ---------------------------------------- softmax: warps 2-5 tile a, 6-9 tile b
+    const int t = (warp - 2) >> 2;
     const int q = warp & 3;
-    const int r = q * 32 + lane;                      // query row within the tile == TMEM lane
+    const int r = q * 32 + lane;  // row within the query tile == TMEM lane
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    const uint32_t s_addr = tmem + lane_base + C::S_COL + t * kBKV;
+    const uint32_t o_addr = tmem + lane_base + C::O_COL + t * 128;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
-      const int sb = j & 1;
-      if (!mbar_wait(&s_full[sb], (j >> 1) & 1)) { ok = false; break; }
+      if (!mbar_wait(&s_full[t], j & 1)) { ok = false; break; }
+      // consume pv_done_t phase j-1 (already complete: s_full_t(j) is committed
+      // after PV_t(j-1)) so that the final parity wait is never two phases ahead
+      if (j > 0 && !mbar_wait(&pv_done[t], (j - 1) & 1)) { ok = false; break; }
       tc_fence_after();
       float s[kBKV];
 #pragma unroll
-      for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(tmem + lane_base + sb * kBKV + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
+      for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
       tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&s_free[sb]);
       const int64_t kv0 = (int64_t)j * kBKV;
       float mx = -INFINITY;
       if (kv0 + kBKV <= a.nk) {
@@ -199,63 +211,59 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           mx = fmaxf(mx, s[i]);
         }
       }
+      // s_full_t(j) is committed after PV_t(j-1), so O_t and the P_t region are
+      // free here.  Lazy rescaling: keep the reference max unless it grew by 2^8.
+      bool resc = false;
+      float f = 1.0f;
       if (j > 0) {
-        // PV_{j-1} must be done before O is rescaled or the P buffer reused
-        if (!mbar_wait(pv_done, (j - 1) & 1)) { ok = false; break; }
-        tc_fence_after();
-        const bool resc = mx > m_run + kRescaleLog2;
-        if (__any_sync(0xffffffffu, resc)) {
-          const float f = resc ? ex2_approx(m_run - mx) : 1.0f;
-#pragma unroll 1
-          for (int c = 0; c < D; c += 32) {
-            uint32_t o[32];
-            tmem_ld32(tmem + lane_base + C::O_COL + c, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
-            tmem_st32(tmem + lane_base + C::O_COL + c, o);
-          }
-          tmem_wait_st();
-          if (resc) {
-            l_run *= f;
-            m_run = mx;
-          }
+        resc = mx > m_run + kRescaleLog2;
+        if (resc) {
+          f = ex2_approx(m_run - mx);
+          l_run *= f;
+          m_run = mx;
         }
       } else {
         m_run = mx;
       }
-      // P = 2^(s - m_run), stored as bf16 in the 128-byte-swizzled K-major layout
+      // P = 2^(s - m_run) as bf16 pairs over the first 64 columns of S_t
       float ls = 0.f;
 #pragma unroll
-      for (int c8 = 0; c8 < kBKV / 8; ++c8) {
-        float p[8];
+      for (int half = 0; half < 2; ++half) {
+        uint32_t pk[32];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          p[i] = ex2_approx(s[c8 * 8 + i] - m_run);
-          ls += p[i];
+        for (int i = 0; i < 32; ++i) {
+          const float p0 = ex2_approx(s[half * 64 + 2 * i] - m_run);
+          const float p1 = ex2_approx(s[half * 64 + 2 * i + 1] - m_run);
+          ls += p0 + p1;
+          pk[i] = pack_bf16(p0, p1);
         }
-        uint4 u;
-        u.x = pack_bf16(p[0], p[1]);
-        u.y = pack_bf16(p[2], p[3]);
-        u.z = pack_bf16(p[4], p[5]);
-        u.w = pack_bf16(p[6], p[7]);
-        const int chunk = c8 >> 3, unit = c8 & 7;
-        *reinterpret_cast<uint4*>(sP + chunk * C::CHUNK_BYTES + r * 128 + ((unit ^ (r & 7)) << 4)) = u;
+        tmem_st32(s_addr + half * 32, pk);
       }
       l_run += ls;
-      fence_proxy_async_smem();
+      if (__any_sync(0xffffffffu, resc)) {
+#pragma unroll 1
+        for (int c = 0; c < D; c += 32) {
+          uint32_t o[32];
+          tmem_ld32(o_addr + c, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+          tmem_st32(o_addr + c, o);
+        }
+      }
+      tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(p_full);
+      mbar_arrive(&p_full[t]);
     }
-    // ---------------------------------------------------- epilogue: O / l
-    if (ok) ok = mbar_wait(pv_done, (nkv - 1) & 1);
+    // ---------------------------------------------------- epilogue: O_t / l
+    if (ok) ok = mbar_wait(&pv_done[t], (nkv - 1) & 1);
     tc_fence_after();
-    const int64_t row = (int64_t)qt * kBQ + r;
+    const int64_t row = (int64_t)qt * kBQ + t * kTileQ + r;
     const float inv = 1.0f / l_run;
 #pragma unroll 1
     for (int c = 0; c < D; c += 32) {
       uint32_t o[32];
-      tmem_ld32(tmem + lane_base + C::O_COL + c, o);
+      tmem_ld32(o_addr + c, o);
       tmem_wait_ld();
       if (ok && row < a.nq) {
         float v[32];
@@ -284,7 +292,7 @@ acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
     attr_done = true;
   }
   CUtensorMap tq, tk, tv;
-  ACID_TRY(make_tmap_bf16(&tq, x.q, x.nq, x.ldq, x.ldq, kBQ));
+  ACID_TRY(make_tmap_bf16(&tq, x.q, x.nq, x.ldq, x.ldq, kTileQ));
   ACID_TRY(make_tmap_bf16(&tk, x.k, x.nk, x.ldk, x.ldk, kBKV));
   ACID_TRY(make_tmap_bf16(&tv, x.v, x.nk, x.ldv, x.ldv, kBKV));
   AttnDev a;
