@@ -48,6 +48,7 @@ BlockWs block_ws_layout(const acid_block_desc& d, void* base) {
   const int64_t att_cols = d.kind == ACID_BLOCK_HV_SINGLE ? (int64_t)d.d + d.ffn : d.d;
   w.att = b.take<uint8_t>(rows * att_cols * es);
   w.hid = d.kind == ACID_BLOCK_HV_SINGLE ? nullptr : b.take<uint8_t>(rows * (int64_t)d.ffn * es);
+  w.xm = d.kind == ACID_BLOCK_HV_SINGLE ? nullptr : b.take<float>(rows * (int64_t)d.d);
   w.kvc = (d.kind == ACID_BLOCK_WAN && d.n_text > 0) ? b.take<uint8_t>(d.n_text * 2 * (int64_t)d.d * es) : nullptr;
   w.bytes = b.off + 1024;
   return w;
@@ -170,7 +171,29 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
     return ACID_OK;
   }
 
-  // ---- attention branch: x += g1 * O(Attn(RoPE(QKV(LNmod1 x))))
+  // The residual stream between the two branches is kept in fp32 (xm): the
+  // attention branch writes x + g1 * (...) to xm, cross-attention adds into
+  // xm, and the FFN branch writes the final x = xm + g2 * (...) in the block
+  // dtype, so a bf16 block rounds its residual stream once.
+  float* xm = ws.xm;
+  auto gated_to_xm = [&](int64_t r0) {  // out: xm, residual: x (block dtype)
+    Epilogue e = gated(2);
+    e.row_base = r0;
+    e.residual = off(x, r0 * d, dt);
+    e.res_fp32 = dt == ACID_FP32;
+    e.out_fp32 = true;
+    return e;
+  };
+  auto gated_from_xm = [&](int64_t r0) {  // out: x (block dtype), residual: xm
+    Epilogue e = gated(5);
+    e.row_base = r0;
+    e.residual = xm + r0 * d;
+    e.res_fp32 = true;
+    e.out_fp32 = dt == ACID_FP32;
+    return e;
+  };
+
+  // ---- attention branch: xm = x + g1 * O(Attn(RoPE(QKV(LNmod1 x))))
   ACID_TRY(ln_mod(dt, x, dt, ws.u, rows, d, mv, mv + d, mt, mt + d, L, eps, s));
   if (D.kind == ACID_BLOCK_HV_DUAL) {
     Epilogue et = ep_qkv;
@@ -185,19 +208,15 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
   self.ldo = d;
   ACID_TRY(attention_forward(dt, self, s));
   if (D.kind == ACID_BLOCK_HV_DUAL) {
-    Epilogue et = gated(2);
-    ACID_TRY(lin(dt, ws.att, d, L, d, W.t_o, d, x, d, et, s));
-    Epilogue ev = gated(2);
-    ev.row_base = L;
-    ev.residual = off(x, L * d, dt);
-    ACID_TRY(lin(dt, off(ws.att, L * d, dt), d, Nv, d, W.o, d, off(x, L * d, dt), d, ev, s));
+    ACID_TRY(lin(dt, ws.att, d, L, d, W.t_o, d, xm, d, gated_to_xm(0), s));
+    ACID_TRY(lin(dt, off(ws.att, L * d, dt), d, Nv, d, W.o, d, xm + L * d, d, gated_to_xm(L), s));
   } else {
-    ACID_TRY(lin(dt, ws.att, d, rows, d, W.o, d, x, d, gated(2), s));
+    ACID_TRY(lin(dt, ws.att, d, rows, d, W.o, d, xm, d, gated_to_xm(0), s));
   }
 
-  // ---- cross-attention (WAN with text): x += O_c(Attn(Q_c(LN x), KV_c(ctx)))
+  // ---- cross-attention (WAN with text): xm += O_c(Attn(Q_c(LN xm), KV_c(ctx)))
   if (D.kind == ACID_BLOCK_WAN && D.n_text > 0) {
-    ACID_TRY(ln_mod(dt, x, dt, ws.u, rows, d, nullptr, nullptr, nullptr, nullptr, 0, eps, s));
+    ACID_TRY(ln_mod(ACID_FP32, xm, dt, ws.u, rows, d, nullptr, nullptr, nullptr, nullptr, 0, eps, s));
     Epilogue eb;
     ACID_TRY(lin(dt, ws.u, d, rows, d, W.cq, d, ws.att, d, eb, s));
     ACID_TRY(lin(dt, ctx, d, D.n_text, d, W.ckv, 2 * d, ws.kvc, 2 * d, eb, s));
@@ -217,27 +236,25 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
     ACID_TRY(attention_forward(dt, cross, s));
     Epilogue er;
     er.kind = EPI_RES;
-    er.residual = x;
+    er.residual = xm;
     er.ldr = d;
-    ACID_TRY(lin(dt, ws.u, d, rows, d, W.co, d, x, d, er, s));
+    er.res_fp32 = true;
+    er.out_fp32 = true;
+    ACID_TRY(lin(dt, ws.u, d, rows, d, W.co, d, xm, d, er, s));
   }
 
-  // ---- FFN branch: x += g2 * W2 GELU(W1 LNmod2 x)
-  ACID_TRY(ln_mod(dt, x, dt, ws.u, rows, d, mv + 3 * d, mv + 4 * d, mt + 3 * d, mt + 4 * d, L, eps, s));
+  // ---- FFN branch: x = xm + g2 * W2 GELU(W1 LNmod2 xm)
+  ACID_TRY(ln_mod(ACID_FP32, xm, dt, ws.u, rows, d, mv + 3 * d, mv + 4 * d, mt + 3 * d, mt + 4 * d, L, eps, s));
   Epilogue eg;
   eg.kind = EPI_GELU;
   if (D.kind == ACID_BLOCK_HV_DUAL) {
     ACID_TRY(lin(dt, ws.u, d, L, d, W.t_ff1, F, ws.hid, F, eg, s));
     ACID_TRY(lin(dt, off(ws.u, L * d, dt), d, Nv, d, W.ff1, F, off(ws.hid, L * F, dt), F, eg, s));
-    Epilogue et = gated(5);
-    ACID_TRY(lin(dt, ws.hid, F, L, F, W.t_ff2, d, x, d, et, s));
-    Epilogue ev = gated(5);
-    ev.row_base = L;
-    ev.residual = off(x, L * d, dt);
-    ACID_TRY(lin(dt, off(ws.hid, L * F, dt), F, Nv, F, W.ff2, d, off(x, L * d, dt), d, ev, s));
+    ACID_TRY(lin(dt, ws.hid, F, L, F, W.t_ff2, d, x, d, gated_from_xm(0), s));
+    ACID_TRY(lin(dt, off(ws.hid, L * F, dt), F, Nv, F, W.ff2, d, off(x, L * d, dt), d, gated_from_xm(L), s));
   } else {
     ACID_TRY(lin(dt, ws.u, d, rows, d, W.ff1, F, ws.hid, F, eg, s));
-    ACID_TRY(lin(dt, ws.hid, F, rows, F, W.ff2, d, x, d, gated(5), s));
+    ACID_TRY(lin(dt, ws.hid, F, rows, F, W.ff2, d, x, d, gated_from_xm(0), s));
   }
   return ACID_OK;
 }

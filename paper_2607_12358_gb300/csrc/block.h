@@ -31,6 +31,7 @@ struct BlockWs {
   uint8_t* att = nullptr;  // [rows, d] (HV_SINGLE: [rows, d + ffn])
   uint8_t* hid = nullptr;  // [rows, ffn]
   uint8_t* kvc = nullptr;  // [n_text, 2d] cross-attention keys / values
+  float* xm = nullptr;     // [rows, d] fp32 residual stream between the two branches
   size_t bytes = 0;
 };
 

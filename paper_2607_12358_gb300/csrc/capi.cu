@@ -186,6 +186,7 @@ extern "C" acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t
   e.residual = residual;
   e.ldr = ldr;
   e.out_fp32 = out_fp32 != 0 || dtype == ACID_FP32;
+  e.res_fp32 = e.out_fp32;  // the residual has the output's dtype
   return linear_forward(dtype, A, lda, M, K, W, N, out, ldo, e, (cudaStream_t)stream);
 }
 

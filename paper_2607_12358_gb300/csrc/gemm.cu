@@ -31,6 +31,7 @@ struct EpiDev {
   int64_t gate_split;
   const void* res;
   int64_t ldr;
+  int res_fp32;
   int64_t row_base;
   RopeTable rope;
   int64_t rope_first_video;
@@ -46,6 +47,7 @@ EpiDev to_dev(const Epilogue& e) {
   d.gate_split = e.gate_split;
   d.res = e.residual;
   d.ldr = e.ldr;
+  d.res_fp32 = e.res_fp32 ? 1 : 0;
   d.row_base = e.row_base;
   d.rope = e.rope;
   d.rope_first_video = e.rope_first_video;
@@ -147,7 +149,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
   float rv[32];
   if (epi_reads_res(e.kind)) {
-    if (g.out_fp32) {
+    if (e.res_fp32) {
       const float* rp = static_cast<const float*>(e.res) + row * e.ldr + col0;
 #pragma unroll
       for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);

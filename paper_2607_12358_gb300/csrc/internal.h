@@ -41,6 +41,7 @@ struct Epilogue {
   int64_t gate_split = 0;
   const void* residual = nullptr;  // [M, ldr] (may equal out)
   int64_t ldr = 0;
+  bool res_fp32 = false;           // residual dtype fp32 (else the GEMM dtype)
   int64_t row_base = 0;            // global row index of GEMM row 0
   // rope: columns [0, 2d) hold q then k; video rows are global rows >= rope_first_video
   RopeTable rope;

@@ -1,0 +1,172 @@
+"""Full-size checks on the workloads' real shapes (through the C ABI).
+
+* One full-length block per block kind: Wan-2.1-1.3B (32760 video tokens,
+  cross-attention to 512 text tokens), CogVideoX-2B (226 + 17550 tokens, head
+  dim 64), HunyuanVideo dual- and single-stream (256 + 67320 tokens, d=3072).
+  The GPU computes every row; the oracle computes sampled rows one by one
+  (keys and values for all tokens), including text rows and the ragged last
+  128-row tile.
+* One sampler step at the Wan shape (one block deep so the oracle can follow):
+  the drift signal teacher-forced from the GPU's own latents, the decision
+  replayed through the oracle controller, and the latent update of a computed
+  and of a forced-skip (cached residual) step at sampled tokens.
+* One EasyCache step at the Cog shape: the signal k mean|dx| / mean|v_prev|
+  recomputed from the GPU latent trajectory.
+"""
+
+import numpy as np
+import pytest
+
+import acid_synth as S
+import oracle as O
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def acid():
+    import __graft_entry__ as g
+
+    g.build()
+    from paper_2607_12358_gb300 import acid as a
+
+    return a
+
+
+def _rows(n_total, n_text, seed=0):
+    rng = np.random.default_rng(seed)
+    base = {0, 1, 2, 3, n_total - 1, n_total - 2, n_total - 3, n_total - 4, n_total - 60, n_total - 127}
+    if n_text:
+        base |= {n_text - 1, n_text, n_text + 1, n_text // 2}
+    base |= set(rng.integers(0, n_total, size=24).tolist())
+    return np.array(sorted(r for r in base if 0 <= r < n_total))
+
+
+def _check(got, ref, x):
+    rel = np.linalg.norm(got - ref) / np.linalg.norm(ref)
+    assert rel <= 1e-2, rel
+    err = np.abs(got - ref)
+    i = np.unravel_index(np.argmax(err), err.shape)
+    assert err.max() <= 5e-2, (err.max(), i, float(ref[i]), float(x[i]))
+    floor = np.linalg.norm(S.round_to_bf16(ref.astype(np.float32)) - ref)
+    assert np.linalg.norm(got - ref) <= 3 * floor + 2e-2 * np.linalg.norm(ref - x)
+
+
+def _gpu_block(acid, cfg, bt, w, x, temb, ctx=None):
+    blk = acid.DeviceBlock.upload(w, bt, torch.bfloat16, DEV)
+    tx = torch.from_numpy(x).to(DEV, torch.bfloat16)
+    acid.acid_dit_block_forward(acid.block_desc(cfg, bt), tx, torch.from_numpy(temb).to(DEV), blk,
+                                ctx=None if ctx is None else torch.from_numpy(ctx).to(DEV, torch.bfloat16))
+    torch.cuda.synchronize()
+    acid.check_device_error()
+    out = tx.float().cpu().numpy()
+    del tx, blk
+    torch.cuda.empty_cache()
+    return out
+
+
+@pytest.mark.parametrize("name,bt", [("wan", "wan"), ("cog", "cog"), ("hv", "hv_dual"), ("hv", "hv_single")])
+def test_full_length_block(acid, name, bt):
+    cfg = S.get_config(name)
+    w = S.block_weights(cfg, 0, seed=11, block_type=bt)
+    L = 0 if bt == "wan" else cfg.n_text
+    n = cfg.n_video + L
+    x = S.hidden(cfg, n, seed=11)
+    # the workload's own timestep embedding (time MLP of the random-weight model at t = 500)
+    temb = O.time_embedding(500.0, S.model_weights(cfg, 11, blocks=False), cfg.time_freq_dim).astype(np.float32)
+    ctx = S.round_to_bf16(S.normal(11, (cfg.n_text, cfg.d), 1.0, "full", "ctx")) if bt == "wan" else None
+    got = _gpu_block(acid, cfg, bt, w, x, temb, ctx)
+    rows = _rows(n, L)
+    if bt == "wan":
+        ref = O.wan_block(x, O.block_modulation(temb, w["mod"]), w, cfg.grid, cfg.heads, ctx=ctx, rows=rows)
+    elif bt == "cog":
+        ref = O.cog_block(x, O.block_modulation(temb, w["mod"]), w, cfg.grid, cfg.heads, L, rows=rows)
+    elif bt == "hv_single":
+        ref = O.hv_single_block(x, O.block_modulation(temb, w["mod"]), w, cfg.grid, cfg.heads, L, rows=rows)
+    else:
+        rt, rv = rows[rows < L], rows[rows >= L] - L
+        yt, yv = O.hv_dual_block(x[:L], x[L:], O.block_modulation(temb, w["txt.mod"]),
+                                 O.block_modulation(temb, w["vid.mod"]), w, cfg.grid, cfg.heads,
+                                 rows_vid=rv, rows_txt=rt)
+        ref = np.concatenate([yt, yv])
+    _check(got[rows], ref, x[rows])
+
+
+def _token_positions(cfg, tokens):
+    """Latent indices (c, f, h, w) covered by the given video tokens."""
+    F_, H, W = cfg.grid
+    out = []
+    for n in tokens:
+        f, h, w = n // (H * W), (n // W) % H, n % W
+        for c in range(cfg.latent_c):
+            for dh in range(cfg.ph):
+                for dw in range(cfg.pw):
+                    out.append((c, f * cfg.pt, h * cfg.ph + dh, w * cfg.pw + dw))
+    return tuple(np.array(out).T)
+
+
+def test_wan_step_drift_decision_and_apply(acid):
+    cfg = S.get_config("wan", n_blocks=1, steps=50)
+    w = S.model_weights(cfg, 21)
+    lat = S.latent(cfg, 21)
+    text = S.text(cfg, 21)
+    model = acid.DeviceModel(cfg, w, DEV)
+    # step 0 computes (warmup), step 1 is forced to reuse the cached residual
+    c, keep = acid.loop_cfg(cfg, n_steps=cfg.steps, forced=[None, False] + [None] * (cfg.steps - 2))
+    loop = acid.Loop(model, c, torch.from_numpy(text).to(DEV, torch.bfloat16), DEV)
+    tl = torch.from_numpy(lat).to(DEV)
+    xs, logs = [tl.cpu().numpy().astype(np.float64)], []
+    for _ in range(2):
+        logs.append(acid.log_to_dict(loop.step(tl)))
+        xs.append(tl.cpu().numpy().astype(np.float64))
+    acid.check_device_error()
+    assert [l["computed"] for l in logs] == [1, 0]
+    sig = O.sigmas(cfg.steps)
+    ctx = O.text_context(cfg, w, text)
+    # (1) signal teacher-forced from the GPU latents
+    si = [O.step_inputs(cfg, w, xs[i], 1000 * sig[i]) for i in range(2)]
+    temni = [O.block0_temni(cfg, w, si[i].h_in, si[i].temb) for i in range(2)]
+    s_ref = O.rel_l1(temni[0], temni[1])
+    assert abs(logs[1]["signal"] - s_ref) <= 1e-3 * s_ref
+    # (2) the natural decision on that signal (oracle controller replay)
+    skip, tau, sg, _ = O.AcidController(cfg.tau_low, cfg.tau_high, cfg.delta).step(logs[1]["signal"])
+    assert logs[1]["tau"] == tau and logs[1]["sigma"] == pytest.approx(sg)
+    # (3) computed step 0 and (4) reused step 1 at sampled tokens
+    tokens = np.array(sorted({0, 1, 777, 16000, cfg.n_video - 1, cfg.n_video - 100}))
+    ref_blk = O.wan_block(si[0].h_in, si[0].mods[0], w["blocks"][0], cfg.grid, cfg.heads, ctx=ctx, rows=tokens)
+    R0 = ref_blk - si[0].h_in[tokens]
+    pos = _token_positions(cfg, tokens)
+    for i, h_out in ((0, ref_blk), (1, si[1].h_in[tokens] + R0)):
+        fm = si[i].final_mod
+        y = O.modulate(O.layer_norm(h_out), fm[:cfg.d], fm[cfg.d:])
+        # [tokens, C*pt*ph*pw] with features ordered (c, dt, dh, dw); pt = 1, so the
+        # flattened order matches _token_positions' (token, c, dh, dw) order
+        v_ref = O.linear(y, *w["final"]).reshape(-1)
+        v_gpu = (xs[i + 1][pos] - xs[i][pos]) / (sig[i + 1] - sig[i])
+        rel = np.linalg.norm(v_gpu - v_ref) / np.linalg.norm(v_ref)
+        assert rel <= 2e-2, (i, rel)
+
+
+def test_cog_easycache_step_signal(acid):
+    cfg = S.get_config("cog", n_blocks=1, steps=50)
+    w = S.model_weights(cfg, 31)
+    lat = S.latent(cfg, 31)
+    text = S.text(cfg, 31)
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg, n_steps=cfg.steps)
+    loop = acid.Loop(model, c, torch.from_numpy(text).to(DEV, torch.bfloat16), DEV)
+    tl = torch.from_numpy(lat).to(DEV)
+    xs, logs = [tl.cpu().numpy().astype(np.float64)], []
+    for _ in range(3):
+        logs.append(acid.log_to_dict(loop.step(tl)))
+        xs.append(tl.cpu().numpy().astype(np.float64))
+    acid.check_device_error()
+    sig = O.sigmas(cfg.steps)
+    v = [(xs[i + 1] - xs[i]) / (sig[i + 1] - sig[i]) for i in range(3)]
+    k = O.easycache_rate(xs[1], xs[0], v[1], v[0])
+    s_ref = O.easycache_signal(k, xs[2], xs[1], v[1])
+    assert abs(logs[2]["signal"] - s_ref) <= 1e-3 * s_ref, (logs[2]["signal"], s_ref)
+    skip, tau, sg, _ = O.AcidController(cfg.tau_low, cfg.tau_high, cfg.delta).step(logs[2]["signal"])
+    assert bool(logs[2]["computed"]) == (not skip)
