@@ -118,6 +118,23 @@ acid_status acid_drift_signal(const void* prev, const void* cur, int64_t n, int3
 acid_status acid_cache_apply(const void* x, const void* cached_residual, void* out, int64_t n,
                              int32_t dtype, acid_stream_t stream);
 
+/* acid_drift_signal without a workspace, for callers that cannot allocate
+ * any device memory: for example a plugin that is handed only its input and
+ * output buffers by a host framework, or a process whose device memory is
+ * fully reserved by another allocator.  The paper has no counterpart: this is
+ * a deployment variant of the drift reduction above, with the same result.
+ *   Arguments and outputs as acid_drift_signal (device or host outputs).
+ *   n          0 <= n <= 2^33; larger n fails with ACID_ERR_UNSUPPORTED.
+ * Scratch: a 16 KiB array in the library's device memory, held by every GPU
+ * that loads the library until the process exits.  No cudaMalloc, cudaFree
+ * or allocating library call is made.  The first call on each device looks
+ * up the array's device address (cudaGetSymbolAddress); make that first call
+ * outside any stream capture.  All calls share the array and it keeps the
+ * last call's contents: calls that overlap on the GPU (different streams
+ * without ordering) race and give undefined results. */
+acid_status acid_drift_signal_noalloc(const void* prev, const void* cur, int64_t n, int32_t dtype,
+                                      double* out_rel_l1, double* out_sums, acid_stream_t stream);
+
 /* Drift and reuse in one pass over HBM (the two calls above fused):
  * rel_l1(prev, cur) as acid_drift_signal and out = cur + cached_residual.
  * Same argument rules; out may alias cur or cached_residual. */

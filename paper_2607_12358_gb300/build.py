@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libacid_gb300.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["capi.cu", "elementwise.cu", "gemm.cu", "attention.cu", "block.cu", "loop.cu"]
+SOURCES = ["capi.cu", "elementwise.cu", "gemm.cu", "attention.cu", "block.cu", "loop.cu", "noalloc.cu"]
 
 
 def nvcc() -> str:
