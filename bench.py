@@ -38,6 +38,21 @@ WORKLOAD = ("Wan-2.1-1.3B-shaped 480p step: 30 blocks, d=1536, 12 heads x 128, F
 CPU_SAMPLE_ROWS = 4096
 REF_SAMPLE_ROWS = 2048
 
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one ncu capture of a
+# self- and a cross-attention launch at this shape) per attention launch of
+# the step's 1:1 self/cross mix.  Valid only for the kernel source it was
+# measured on; any other source reports null.
+ATTN_TRAFFIC = {"source_sha256_16": "22ef4ab31cc592f1", "bytes_per_launch": (393.26e6 + 155.95e6) / 2}
+
+
+def _attn_traffic():
+    import hashlib
+
+    src = os.path.join(ROOT, "paper_2607_12358_gb300", "csrc", "attention.cu")
+    with open(src, "rb") as f:
+        h = hashlib.sha256(f.read()).hexdigest()[:16]
+    return ATTN_TRAFFIC["bytes_per_launch"] if h == ATTN_TRAFFIC["source_sha256_16"] else None
+
 
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
@@ -306,7 +321,7 @@ def run_ours(args) -> None:
                    "l2": "no flush: per-step working set (2.8 GB weights, >0.5 GB activations) exceeds the 129 MB L2"},
         "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel<128> (self + cross attention)",
                      "achieved": att_tflops, "peak": peak, "unit": "TFLOP/s", "frac": att_tflops / peak,
-                     "peak_source": f"bf16_tflops_sustained, {src}", "traffic": None,
+                     "peak_source": f"bf16_tflops_sustained, {src}", "traffic": _attn_traffic(),
                      "frac_of_burst_peak": att_tflops / peaks["bf16_tflops"],
                      "launches": a_n, "avg_launch_ms": a_ms / max(a_n, 1)},
         "attention_tflops": att_tflops,
