@@ -128,7 +128,9 @@ struct TcCfg {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr int EPI_STAGE_FLOATS = 32 * 33;  // one 32x32 chunk per epilogue warp, padded rows
+  static constexpr int EPI_BYTES = kEpiWarps * EPI_STAGE_FLOATS * 4;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + EPI_BYTES + 1024 + 256;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -140,42 +142,97 @@ struct GemmDims {
   int out_fp32;
 };
 
-template <int BN>
-__device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, int64_t row, int col0,
-                                               const uint32_t* r) {
-  const int64_t grow = row + e.row_base;
-  float v[32];
+// Epilogue of 32-row x 32-column accumulator chunks held by a warp (thread =
+// row after tcgen05.ld).  Each chunk is transposed through shared memory so
+// that every global access of the warp covers whole row segments: lane l
+// handles columns 4(l%8) .. 4(l%8)+3 of rows 4p + l/8, p = 0..7.  Residual
+// values of the next chunk are loaded while the current one is processed, so
+// each lane keeps up to 16 loads in flight.
+struct ResChunk {
+  float v[8][4];
+};
+
+__device__ __forceinline__ void load_res_chunk(const GemmDims& g, const EpiDev& e, int64_t row0, int col,
+                                               ResChunk& rc) {
+  const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-  float rv[32];
-  if (epi_reads_res(e.kind)) {
+  for (int p = 0; p < 8; ++p) {
+    const int64_t row = row0 + 4 * p + (lane >> 3);
+    if (row >= g.M) continue;
     if (e.res_fp32) {
-      const float* rp = static_cast<const float*>(e.res) + row * e.ldr + col0;
-#pragma unroll
-      for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
+      const float4 t = *reinterpret_cast<const float4*>(static_cast<const float*>(e.res) + row * e.ldr + col);
+      rc.v[p][0] = t.x; rc.v[p][1] = t.y; rc.v[p][2] = t.z; rc.v[p][3] = t.w;
     } else {
-      const __nv_bfloat16* rp = static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col0;
-#pragma unroll
-      for (int j = 0; j < 32; j += 8) load8(rp + j, rv + j);
+      const uint2 t = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col);
+      rc.v[p][0] = bf16_lo(t.x); rc.v[p][1] = bf16_hi(t.x); rc.v[p][2] = bf16_lo(t.y); rc.v[p][3] = bf16_hi(t.y);
     }
-  } else {
-#pragma unroll
-    for (int j = 0; j < 32; ++j) rv[j] = 0.f;
-  }
-#pragma unroll
-  for (int j = 0; j < 32; j += 2) epi_pair<true>(e, grow, col0 + j, v[j], v[j + 1], rv[j], rv[j + 1]);
-  if (g.out_fp32) {
-    float* op = static_cast<float*>(g.out) + row * g.ldo + col0;
-#pragma unroll
-    for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
-  } else {
-    __nv_bfloat16* op = static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col0;
-#pragma unroll
-    for (int j = 0; j < 32; j += 8) store8(op + j, v + j);
   }
 }
 
-template <int BN>
+template <int KIND>
+__device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, float* stage, int64_t row0,
+                                               int col0, const uint32_t* r, const ResChunk& rc) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int j = 0; j < 32; ++j) stage[lane * 33 + j] = __uint_as_float(r[j]);
+  __syncwarp();
+  const int c = 4 * (lane & 7);
+  const int col = col0 + c;
+  float bias[4], gv[4], gt[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    bias[k] = e.bias ? e.bias[col + k] : 0.f;
+    gv[k] = KIND == EPI_GATED_RES ? e.gate_v[col + k] : 0.f;
+    gt[k] = KIND == EPI_GATED_RES ? e.gate_t[col + k] : 0.f;
+  }
+#pragma unroll
+  for (int p = 0; p < 8; ++p) {
+    const int rr = 4 * p + (lane >> 3);
+    const int64_t row = row0 + rr;
+    if (row >= g.M) continue;
+    const int64_t grow = row + e.row_base;
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = stage[rr * 33 + c + k] + bias[k];
+    switch (KIND) {
+      case EPI_GELU:
+#pragma unroll
+        for (int k = 0; k < 4; ++k) v[k] = gelu_tanh<true>(v[k]);
+        break;
+      case EPI_ROPE_QKV:
+        if (col < 2 * e.d && grow >= e.rope_first_video) {
+#pragma unroll
+          for (int k = 0; k < 4; k += 2) {
+            const float2 cs = rope_cs(e.rope, grow - e.rope_first_video, ((col + k) % e.head_dim) >> 1);
+            const float x0 = v[k], x1 = v[k + 1];
+            v[k] = x0 * cs.x - x1 * cs.y;
+            v[k + 1] = x0 * cs.y + x1 * cs.x;
+          }
+        }
+        break;
+      case EPI_GATED_RES: {
+        const bool text = grow < e.gate_split;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) v[k] = fmaf(text ? gt[k] : gv[k], v[k], rc.v[p][k]);
+        break;
+      }
+      case EPI_RES:
+#pragma unroll
+        for (int k = 0; k < 4; ++k) v[k] += rc.v[p][k];
+        break;
+      default:
+        break;
+    }
+    if (g.out_fp32)
+      *reinterpret_cast<float4*>(static_cast<float*>(g.out) + row * g.ldo + col) = make_float4(v[0], v[1], v[2], v[3]);
+    else
+      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col) =
+          make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
+  }
+  __syncwarp();
+}
+
+template <int BN, int KIND>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
                    EpiDev e) {
@@ -184,7 +241,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES + C::EPI_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* acc_full = empty + C::STAGES;  // [2]
   uint64_t* acc_empty = acc_full + 2;      // [2]
@@ -259,21 +316,35 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   } else {  // epilogue: warps 2..9; lane quarter = warp % 4, column half = (warp - 2) / 4
     const int q = warp & 3, half = (warp - 2) >> 2;
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    float* stage = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES) + (warp - 2) * C::EPI_STAGE_FLOATS;
     int local = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
       const int b = local & 1, use = local >> 1;
       const int m_tile = tile / num_n, n_tile = tile % num_n;
       const bool ok = mbar_wait(&acc_full[b], use & 1);
       tc_fence_after();
-      const int64_t row = (int64_t)m_tile * BM + q * 32 + lane;
-      const bool row_ok = ok && row < g.M;
-#pragma unroll 1
-      for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+      const int64_t row0 = (int64_t)m_tile * BM + q * 32;
+      constexpr bool res = KIND == EPI_GATED_RES || KIND == EPI_RES;
+      // this warp's chunks: columns [half * BN/2, (half + 1) * BN/2) of the tile, 32 at a time;
+      // residual values of chunk i+1 are loaded while chunk i is processed
+      constexpr int NC = BN / 64;
+      const int cbeg = half * (BN / 2);
+      const int lcol = 4 * (lane & 7);
+      auto process = [&](int i, const ResChunk& cur, ResChunk& nxt) {
+        const int c = cbeg + 32 * i;
         uint32_t r[32];
         tmem_ld32(tmem + lane_base + b * BN + c, r);
         tmem_wait_ld();
         const int col0 = n_tile * BN + c;
-        if (row_ok && col0 < g.N) epilogue_chunk<BN>(g, e, row, col0, r);
+        if (res && i + 1 < NC && row0 < g.M && col0 + 32 < g.N) load_res_chunk(g, e, row0, col0 + 32 + lcol, nxt);
+        if (ok && row0 < g.M && col0 < g.N) epilogue_chunk<KIND>(g, e, stage, row0, col0, r, cur);
+      };
+      ResChunk rc0, rc1;
+      if (res && row0 < g.M && n_tile * BN + cbeg < g.N) load_res_chunk(g, e, row0, n_tile * BN + cbeg + lcol, rc0);
+#pragma unroll 1
+      for (int i = 0; i < NC; i += 2) {
+        process(i, rc0, rc1);
+        if (i + 1 < NC) process(i + 1, rc1, rc0);
       }
       tc_fence_before();
       mbar_arrive(&acc_empty[b]);
@@ -337,15 +408,23 @@ int num_sms() {
   return n;
 }
 
-template <int BN>
-acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
-                      const Epilogue& epi, cudaStream_t s) {
+template <int BN, int KIND>
+acid_status launch_tc_kind(const CUtensorMap& ta, const CUtensorMap& tb, const GemmDims& g, const Epilogue& epi,
+                           int grid, cudaStream_t s) {
   using C = TcCfg<BN>;
   static bool attr_done = false;
   if (!attr_done) {
-    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN, KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
     attr_done = true;
   }
+  gemm_tc_kernel<BN, KIND><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+template <int BN>
+acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
+                      const Epilogue& epi, cudaStream_t s) {
   CUtensorMap ta, tb;
   ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
   ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, BN));
@@ -353,9 +432,13 @@ acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* 
   const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = (int)std::min<int64_t>(tiles, num_sms());
   ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
-  gemm_tc_kernel<BN><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
-  ACID_CHECK_LAUNCH();
-  return ACID_OK;
+  switch (epi.kind) {
+    case EPI_GELU: return launch_tc_kind<BN, EPI_GELU>(ta, tb, g, epi, grid, s);
+    case EPI_ROPE_QKV: return launch_tc_kind<BN, EPI_ROPE_QKV>(ta, tb, g, epi, grid, s);
+    case EPI_GATED_RES: return launch_tc_kind<BN, EPI_GATED_RES>(ta, tb, g, epi, grid, s);
+    case EPI_RES: return launch_tc_kind<BN, EPI_RES>(ta, tb, g, epi, grid, s);
+    default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, g, epi, grid, s);
+  }
 }
 
 // ===========================================================================
