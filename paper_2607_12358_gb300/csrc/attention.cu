@@ -197,20 +197,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
       tmem_wait_ld();
       const int64_t kv0 = (int64_t)j * kBKV;
-      float mx = -INFINITY;
-      if (kv0 + kBKV <= a.nk) {
+      if (kv0 + kBKV > a.nk) {
 #pragma unroll
-        for (int i = 0; i < kBKV; ++i) {
-          s[i] *= a.scale_log2;
-          mx = fmaxf(mx, s[i]);
-        }
-      } else {
-#pragma unroll
-        for (int i = 0; i < kBKV; ++i) {
-          s[i] = (kv0 + i < a.nk) ? s[i] * a.scale_log2 : -INFINITY;
-          mx = fmaxf(mx, s[i]);
-        }
+        for (int i = 0; i < kBKV; ++i)
+          if (kv0 + i >= a.nk) s[i] = -INFINITY;
       }
+      // row max of the raw scores (four independent 3-input max chains); the
+      // positive scale commutes with max, so it is applied to the max only
+      float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+      for (int i = 0; i < kBKV; i += 8) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) m4[k] = fmax3(m4[k], s[i + 2 * k], s[i + 2 * k + 1]);
+      }
+      const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
       // s_full_t(j) is committed after PV_t(j-1), so O_t and the P_t region are
       // free here.  Lazy rescaling: keep the reference max unless it grew by 2^8.
       bool resc = false;
@@ -225,20 +225,31 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       } else {
         m_run = mx;
       }
-      // P = 2^(s - m_run) as bf16 pairs over the first 64 columns of S_t
-      float ls = 0.f;
+      // P = 2^(s * scale - m_run) as bf16 pairs over the first 64 columns of S_t;
+      // the scale-and-subtract and the row sum run as packed fp32 pairs
+      const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2);
+      const uint64_t nm2 = f2_pack(-m_run, -m_run);
+      uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t pk[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float p0 = ex2_approx(s[half * 64 + 2 * i] - m_run);
-          const float p1 = ex2_approx(s[half * 64 + 2 * i + 1] - m_run);
-          ls += p0 + p1;
+          float e0, e1;
+          f2_unpack(f2_fma(f2_pack(s[half * 64 + 2 * i], s[half * 64 + 2 * i + 1]), sc2, nm2), e0, e1);
+          const float p0 = ex2_approx(e0), p1 = ex2_approx(e1);
+          if (i & 1)
+            acc1 = f2_add(acc1, f2_pack(p0, p1));
+          else
+            acc0 = f2_add(acc0, f2_pack(p0, p1));
           pk[i] = pack_bf16(p0, p1);
         }
         tmem_st32(s_addr + half * 32, pk);
       }
+      float a0, a1, b0, b1;
+      f2_unpack(acc0, a0, a1);
+      f2_unpack(acc1, b0, b1);
+      const float ls = (a0 + a1) + (b0 + b1);
       l_run += ls;
       if (__any_sync(0xffffffffu, resc)) {
 #pragma unroll 1
