@@ -42,7 +42,7 @@ REF_SAMPLE_ROWS = 2048
 # self- and a cross-attention launch at this shape) per attention launch of
 # the step's 1:1 self/cross mix.  Valid only for the kernel source it was
 # measured on; any other source reports null.
-ATTN_TRAFFIC = {"source_sha256_16": "22ef4ab31cc592f1", "bytes_per_launch": (393.26e6 + 155.95e6) / 2}
+ATTN_TRAFFIC = {"source_sha256_16": "e1e6d248900fd9eb", "bytes_per_launch": (404.46e6 + 156.83e6) / 2}
 
 
 def _attn_traffic():
