@@ -171,11 +171,16 @@ acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t lda, int64
 /* Multi-head attention softmax(q k^T / sqrt(head_dim)) v, per head h reading
  * columns [h*head_dim, (h+1)*head_dim) of q (row stride ldq), k (ldk), v (ldv)
  * and writing the same columns of out (ldo).  nq, nk >= 1 rows.  bf16 runs on
- * tcgen05 with head_dim 64 or 128; fp32 with head_dim a multiple of 32, <= 128. */
+ * tcgen05 with head_dim 64 or 128; fp32 with head_dim a multiple of 32, <= 128.
+ *   workspace  optional (NULL, 0): device scratch of
+ *              acid_attention_workspace_size bytes.  With it, the work that
+ *              would run as a last, partly filled wave of CTAs is split along
+ *              the key range and merged (same result up to summation order). */
 acid_status acid_attention_forward(int32_t dtype, const void* q, int64_t ldq, const void* k,
                                    int64_t ldk, const void* v, int64_t ldv, void* out, int64_t ldo,
                                    int64_t nq, int64_t nk, int32_t heads, int32_t head_dim,
-                                   acid_stream_t stream);
+                                   void* workspace, size_t workspace_bytes, acid_stream_t stream);
+acid_status acid_attention_workspace_size(int32_t head_dim, size_t* bytes);
 
 /* adaLN LayerNorm: y = LN(x) * (1 + scale) + shift per row of x [rows, d]
  * (no affine part, epsilon eps); shift / scale fp32 [d] or both NULL.

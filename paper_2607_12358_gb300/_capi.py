@@ -87,7 +87,8 @@ _PROTOS = {
     "acid_linear_forward": (C.c_int, [C.c_int32, _P, C.c_int64, C.c_int64, C.c_int32, _P, _P, C.c_int32, _P,
                                       C.c_int64, C.c_int32, _P, _P, C.c_int64, C.c_int32, _P]),
     "acid_attention_forward": (C.c_int, [C.c_int32, _P, C.c_int64, _P, C.c_int64, _P, C.c_int64, _P, C.c_int64,
-                                         C.c_int64, C.c_int64, C.c_int32, C.c_int32, _P]),
+                                         C.c_int64, C.c_int64, C.c_int32, C.c_int32, _P, C.c_size_t, _P]),
+    "acid_attention_workspace_size": (C.c_int, [C.c_int32, C.POINTER(C.c_size_t)]),
     "acid_layernorm_mod": (C.c_int, [C.c_int32, _P, C.c_int32, _P, C.c_int64, C.c_int32, _P, _P, C.c_float, _P]),
     "acid_block_rows": (C.c_int, [C.POINTER(acid_block_desc), C.POINTER(C.c_int64)]),
     "acid_block_workspace_size": (C.c_int, [C.POINTER(acid_block_desc), C.POINTER(C.c_size_t)]),

@@ -148,15 +148,24 @@ def acid_linear_forward(a: torch.Tensor, w: torch.Tensor, bias: torch.Tensor | N
     return out
 
 
+def attention_workspace_size(head_dim: int) -> int:
+    b = C.c_size_t()
+    check(load().acid_attention_workspace_size(int(head_dim), C.byref(b)))
+    return b.value
+
+
 def acid_attention_forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, heads: int,
-                           out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
-    """softmax(q k^T / sqrt(Dh)) v per head; q [nq, H*Dh], k/v [nk, H*Dh] (row strides taken from the tensors)."""
-    _need_cuda(q, k, v, out)
+                           out: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+                           stream=None) -> torch.Tensor:
+    """softmax(q k^T / sqrt(Dh)) v per head; q [nq, H*Dh], k/v [nk, H*Dh] (row strides taken from the tensors).
+    ``workspace`` (optional, attention_workspace_size bytes) enables the split of a partial last wave."""
+    _need_cuda(q, k, v, out, workspace)
     nq, nk = q.shape[0], k.shape[0]
     hd = q.shape[1] // heads
     out = torch.empty(nq, heads * hd, dtype=q.dtype, device=q.device) if out is None else out
     check(load().acid_attention_forward(_dtype(q), q.data_ptr(), q.stride(0), k.data_ptr(), k.stride(0),
                                         v.data_ptr(), v.stride(0), out.data_ptr(), out.stride(0), nq, nk, heads, hd,
+                                        _ptr(workspace), 0 if workspace is None else workspace.numel(),
                                         _stream(stream)))
     return out
 

@@ -37,6 +37,7 @@ constexpr int kBQ = 2 * kTileQ;
 constexpr int kBKV = 128;  // keys per K/V tile
 constexpr int kAttnThreads = 320;
 constexpr float kRescaleLog2 = 8.0f;
+constexpr int kAttnPartCtas = kAttnSplitCtas;  // CTAs of a split tail wave (partials workspace capacity)
 
 struct AttnDev {
   int64_t nq, nk;
@@ -45,6 +46,15 @@ struct AttnDev {
   int64_t ldo;
   int o_col;
   float scale_log2;  // log2(e) / sqrt(head_dim)
+  // work item = (query-tile pair, head), numbered head-major; CTA blockIdx.x
+  // handles item item_base + blockIdx.x / splits and the split-th part of the
+  // key range.  With splits > 1 the CTA writes its unnormalised output and
+  // (max, sum) per row to part_o / part_ml instead of the final output.
+  int nqp;
+  int item_base;
+  int splits;
+  float* part_o;   // [CTA][256 rows][D]
+  float* part_ml;  // [CTA][256 rows][2]
 };
 
 template <int D>
@@ -85,8 +95,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = blockIdx.x, h = blockIdx.y;
-  const int nkv = (int)((a.nk + kBKV - 1) / kBKV);
+  const int item = a.item_base + (int)blockIdx.x / a.splits, split = (int)blockIdx.x % a.splits;
+  const int qt = item % a.nqp, h = item / a.nqp;
+  const int nkv_all = (int)((a.nk + kBKV - 1) / kBKV);
+  const int jb = (int)((int64_t)split * nkv_all / a.splits);  // this CTA's key tiles [jb, jb + nkv)
+  const int nkv = (int)((int64_t)(split + 1) * nkv_all / a.splits) - jb;
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmQ);
@@ -123,12 +136,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         mbar_expect_tx(&k_full[st], C::T_BYTES);
         for (int c = 0; c < C::CH; ++c)
           tma_load_2d(sK + st * C::T_BYTES + c * C::CHUNK_BYTES, &tmK, &k_full[st], a.k_col + h * D + c * 64,
-                      j * kBKV);
+                      (jb + j) * kBKV);
         if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) break;
         mbar_expect_tx(&v_full[st], C::T_BYTES);
         for (int c = 0; c < C::CH; ++c)
           tma_load_2d(sV + st * C::T_BYTES + c * C::CHUNK_BYTES, &tmV, &v_full[st], a.v_col + h * D + c * 64,
-                      j * kBKV);
+                      (jb + j) * kBKV);
       }
     }
   } else if (warp == 1) {
@@ -196,7 +209,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 #pragma unroll
       for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
       tmem_wait_ld();
-      const int64_t kv0 = (int64_t)j * kBKV;
+      const int64_t kv0 = (int64_t)(jb + j) * kBKV;
       if (kv0 + kBKV > a.nk) {
 #pragma unroll
         for (int i = 0; i < kBKV; ++i)
@@ -276,15 +289,25 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       uint32_t o[32];
       tmem_ld32(o_addr + c, o);
       tmem_wait_ld();
-      if (ok && row < a.nq) {
-        float v[32];
+      if (!ok || row >= a.nq) continue;
+      if (a.splits > 1) {  // partial result of this key range: unnormalised O
+        float* pp = a.part_o + ((int64_t)blockIdx.x * kBQ + t * kTileQ + r) * D + c;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]) * inv;
-        __nv_bfloat16* op = static_cast<__nv_bfloat16*>(a.out) + row * a.ldo + a.o_col + h * D + c;
-#pragma unroll
-        for (int i = 0; i < 32; i += 8) store8(op + i, v + i);
+        for (int i = 0; i < 32; i += 4)
+          *reinterpret_cast<float4*>(pp + i) = make_float4(__uint_as_float(o[i]), __uint_as_float(o[i + 1]),
+                                                           __uint_as_float(o[i + 2]), __uint_as_float(o[i + 3]));
+        continue;
       }
+      float v[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]) * inv;
+      __nv_bfloat16* op = static_cast<__nv_bfloat16*>(a.out) + row * a.ldo + a.o_col + h * D + c;
+#pragma unroll
+      for (int i = 0; i < 32; i += 8) store8(op + i, v + i);
     }
+    if (a.splits > 1 && ok && row < a.nq)
+      *reinterpret_cast<float2*>(a.part_ml + ((int64_t)blockIdx.x * kBQ + t * kTileQ + r) * 2) =
+          make_float2(m_run, l_run);
   }
   tc_fence_before();
   __syncthreads();
@@ -292,6 +315,46 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
+}
+
+// Merges the key-range parts of the split items: for every row,
+// O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s with M = max_s m_s.
+// One warp per row (256 rows per item), D / 32 columns per lane.
+template <int D>
+__global__ void __launch_bounds__(256) attn_merge_kernel(AttnDev a, int item0, int tail, int splits) {
+  const int wrow = (int)(blockIdx.x * 8 + (threadIdx.x >> 5));  // row over all tail items
+  const int lane = threadIdx.x & 31;
+  if (wrow >= tail * kBQ) return;
+  const int it = wrow / kBQ, rr = wrow % kBQ;
+  const int item = item0 + it;
+  const int qt = item % a.nqp, h = item / a.nqp;
+  const int64_t row = (int64_t)qt * kBQ + rr;
+  if (row >= a.nq) return;
+  float M = -INFINITY;
+  for (int sp = 0; sp < splits; ++sp) M = fmaxf(M, a.part_ml[((int64_t)(it * splits + sp) * kBQ + rr) * 2]);
+  float acc[D / 32] = {};
+  float L = 0.f;
+  for (int sp = 0; sp < splits; ++sp) {
+    const int64_t slot = (int64_t)(it * splits + sp) * kBQ + rr;
+    const float w = ex2_approx(a.part_ml[slot * 2] - M);
+    L += w * a.part_ml[slot * 2 + 1];
+#pragma unroll
+    for (int i = 0; i < D / 32; ++i) acc[i] = fmaf(w, a.part_o[slot * D + i * 32 + lane], acc[i]);
+  }
+  const float inv = 1.0f / L;
+  __nv_bfloat16* op = static_cast<__nv_bfloat16*>(a.out) + row * a.ldo + a.o_col + h * D;
+#pragma unroll
+  for (int i = 0; i < D / 32; ++i) op[i * 32 + lane] = __float2bfloat16_rn(acc[i] * inv);
+}
+
+int num_sms_attn() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  }
+  return n;
 }
 
 template <int D>
@@ -316,9 +379,36 @@ acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
   a.ldo = x.ldo;
   a.o_col = x.o_col;
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
-  dim3 grid((unsigned)((x.nq + kBQ - 1) / kBQ), (unsigned)x.heads);
+  a.nqp = (int)((x.nq + kBQ - 1) / kBQ);
+  a.item_base = 0;
+  a.splits = 1;
+  a.part_o = nullptr;
+  a.part_ml = nullptr;
+  const int items = a.nqp * x.heads;
+  const int nkv_all = (int)((x.nk + kBKV - 1) / kBKV);
+  // Items fill whole waves of one CTA per SM; the items of a last, partial
+  // wave are split along the key range so that they fill one wave together,
+  // and their partial results are merged.
+  const int sms = num_sms_attn();
+  const int full = (items / sms) * sms, tail = items - full;
+  int splits = tail > 0 ? std::min(std::min(kAttnPartCtas, sms) / tail, nkv_all) : 1;
+  const size_t part_need = (size_t)tail * splits * kBQ * (D + 2) * sizeof(float);
+  const bool split_tail = full > 0 && tail > 0 && splits >= 2 && x.part != nullptr && x.part_bytes >= part_need;
   ProfScope prof(PROF_ATTENTION, 4.0 * (double)x.nq * (double)x.nk * D * x.heads, s);
-  attn_tc_kernel<D><<<grid, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
+  if (!split_tail) {
+    attn_tc_kernel<D><<<items, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
+    ACID_CHECK_LAUNCH();
+    return ACID_OK;
+  }
+  attn_tc_kernel<D><<<full, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
+  ACID_CHECK_LAUNCH();
+  a.item_base = full;
+  a.splits = splits;
+  a.part_o = static_cast<float*>(x.part);
+  a.part_ml = a.part_o + (size_t)tail * splits * kBQ * D;
+  attn_tc_kernel<D><<<tail * splits, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
+  ACID_CHECK_LAUNCH();
+  attn_merge_kernel<D><<<tail * kBQ / 8, 256, 0, s>>>(a, full, tail, splits);
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }

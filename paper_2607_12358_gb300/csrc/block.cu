@@ -49,6 +49,10 @@ BlockWs block_ws_layout(const acid_block_desc& d, void* base) {
   w.att = b.take<uint8_t>(rows * att_cols * es);
   w.hid = d.kind == ACID_BLOCK_HV_SINGLE ? nullptr : b.take<uint8_t>(rows * (int64_t)d.ffn * es);
   w.xm = d.kind == ACID_BLOCK_HV_SINGLE ? nullptr : b.take<float>(rows * (int64_t)d.d);
+  if (d.dtype == ACID_BF16 && d.heads > 0) {
+    w.attn_part_bytes = attn_part_bytes(d.d / d.heads);
+    w.attn_part = b.take<uint8_t>(w.attn_part_bytes);
+  }
   w.kvc = (d.kind == ACID_BLOCK_WAN && d.n_text > 0) ? b.take<uint8_t>(d.n_text * 2 * (int64_t)d.d * es) : nullptr;
   w.bytes = b.off + 1024;
   return w;
@@ -154,6 +158,8 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
   self.v_col = 2 * d;
   self.nq = self.nk = rows;
   self.heads = D.heads;
+  self.part = ws.attn_part;
+  self.part_bytes = ws.attn_part_bytes;
   self.head_dim = hd;
 
   if (D.kind == ACID_BLOCK_HV_SINGLE) {
@@ -233,6 +239,8 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
     cross.nk = D.n_text;
     cross.heads = D.heads;
     cross.head_dim = hd;
+    cross.part = ws.attn_part;
+    cross.part_bytes = ws.attn_part_bytes;
     ACID_TRY(attention_forward(dt, cross, s));
     Epilogue er;
     er.kind = EPI_RES;

@@ -32,6 +32,8 @@ struct BlockWs {
   uint8_t* hid = nullptr;  // [rows, ffn]
   uint8_t* kvc = nullptr;  // [n_text, 2d] cross-attention keys / values
   float* xm = nullptr;     // [rows, d] fp32 residual stream between the two branches
+  void* attn_part = nullptr;  // attention partial results of a split last wave
+  size_t attn_part_bytes = 0;
   size_t bytes = 0;
 };
 

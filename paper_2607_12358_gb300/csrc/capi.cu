@@ -192,8 +192,11 @@ extern "C" acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t
 
 extern "C" acid_status acid_attention_forward(int32_t dtype, const void* q, int64_t ldq, const void* k, int64_t ldk,
                                               const void* v, int64_t ldv, void* out, int64_t ldo, int64_t nq,
-                                              int64_t nk, int32_t heads, int32_t head_dim, acid_stream_t stream) {
+                                              int64_t nk, int32_t heads, int32_t head_dim, void* workspace,
+                                              size_t workspace_bytes, acid_stream_t stream) {
   clear_error();
+  ACID_REQUIRE(workspace == nullptr || aligned(workspace, 16), ACID_ERR_WORKSPACE,
+               "acid_attention_forward: workspace must be 16-byte aligned");
   ACID_REQUIRE(dtype == ACID_BF16 || dtype == ACID_FP32, ACID_ERR_INVALID_ARG, "acid_attention_forward: unknown dtype");
   ACID_REQUIRE(heads > 0 && head_dim > 0, ACID_ERR_INVALID_ARG, "acid_attention_forward: bad heads / head_dim");
   const int64_t w = (int64_t)heads * head_dim;
@@ -207,7 +210,16 @@ extern "C" acid_status acid_attention_forward(int32_t dtype, const void* q, int6
   a.out = out; a.ldo = ldo;
   a.nq = nq; a.nk = nk;
   a.heads = heads; a.head_dim = head_dim;
+  a.part = workspace;
+  a.part_bytes = workspace ? workspace_bytes : 0;
   return attention_forward(dtype, a, (cudaStream_t)stream);
+}
+
+extern "C" acid_status acid_attention_workspace_size(int32_t head_dim, size_t* bytes) {
+  clear_error();
+  ACID_REQUIRE(bytes != nullptr && head_dim > 0, ACID_ERR_INVALID_ARG, "acid_attention_workspace_size: bad argument");
+  *bytes = attn_part_bytes(head_dim);
+  return ACID_OK;
 }
 
 extern "C" acid_status acid_layernorm_mod(int32_t x_dtype, const void* x, int32_t y_dtype, void* y, int64_t rows,

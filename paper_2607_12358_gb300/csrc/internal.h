@@ -66,8 +66,15 @@ struct AttnArgs {
   void* out = nullptr; int64_t ldo = 0; int o_col = 0;
   int64_t nq = 0, nk = 0;
   int heads = 0, head_dim = 0;
+  // optional scratch for splitting the last partial wave along the key range
+  void* part = nullptr;
+  size_t part_bytes = 0;
 };
 acid_status attention_forward(int dtype, const AttnArgs& a, cudaStream_t s);
+constexpr int kAttnSplitCtas = 160;  // at least the SM count of the target GPU
+inline size_t attn_part_bytes(int head_dim) {
+  return (size_t)kAttnSplitCtas * 256 * (size_t)(head_dim + 2) * sizeof(float);
+}
 
 // ----------------------------------------------------------------- elementwise
 // y[r] = LN(x[r]) * (1 + scale) + shift; rows < split use (shift_t, scale_t).

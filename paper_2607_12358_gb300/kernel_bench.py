@@ -66,7 +66,8 @@ def main():
         qkv = torch.randn(max(a.n, nk), 3 * w, device=dev, generator=gen).to(torch.bfloat16)
         q, k, v = qkv[:a.n, :w], qkv[:nk, w:2 * w], qkv[:nk, 2 * w:]
         o = torch.empty(a.n, w, device=dev, dtype=torch.bfloat16)
-        ms = _time(lambda: acid.acid_attention_forward(q, k, v, a.heads, out=o), a.warmup, a.iters)
+        ws = torch.empty(acid.attention_workspace_size(a.head_dim), dtype=torch.uint8, device=dev)
+        ms = _time(lambda: acid.acid_attention_forward(q, k, v, a.heads, out=o, workspace=ws), a.warmup, a.iters)
         flop = 4.0 * a.n * nk * a.head_dim * a.heads
         out.update(shape=[a.n, nk, a.heads, a.head_dim], ms=ms, tflops=flop / ms / 1e9)
     elif a.kernel == "linear":

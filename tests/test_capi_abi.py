@@ -111,7 +111,9 @@ def test_host_validation_without_gpu(lib):
     assert lib.acid_linear_forward(A.ACID_BF16, None, 64, 10, 64, None, None, 64, None, 64, 9, None, None, 0, 0,
                                    None) == A.ACID_ERR_INVALID_ARG
     assert lib.acid_attention_forward(A.ACID_BF16, None, 64, None, 64, None, 64, None, 64, 0, 4, 1, 64,
-                                      None) == A.ACID_ERR_INVALID_ARG
+                                      None, 0, None) == A.ACID_ERR_INVALID_ARG
+    n = ctypes.c_size_t()
+    assert lib.acid_attention_workspace_size(128, ctypes.byref(n)) == A.ACID_OK and n.value > 0
 
 
 def test_loop_workspace_size_without_gpu(lib):
