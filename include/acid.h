@@ -345,6 +345,22 @@ acid_status acid_denoise_loop(const acid_model* m, const acid_loop_cfg* cfg, voi
                               const void* text, acid_step_log* log, void* workspace,
                               size_t workspace_bytes, acid_stream_t stream);
 
+/* The same generation as acid_denoise_loop, launched as one CUDA graph: a
+ * WHILE node whose body is one sampler step.  The drift signal (TeaCache:
+ * block 0's modulated input and its relative L1 in one fused pass) and
+ * Algorithm 1's decision are computed on the device; the decision selects the
+ * compute or the reuse body of a conditional node, so no step waits for the
+ * host.  Arithmetic and decisions are those of acid_denoise_loop.
+ *   n_steps    <= 1024.
+ *   log        host [n_steps] or NULL; entries as acid_denoise_step writes
+ *              them, with ms = NaN (steps are not timed individually).
+ * Builds, instantiates and launches the graph on `stream`, then synchronises
+ * `stream` and destroys the graph.  CUDA graph objects are created by the
+ * driver for the duration of the call; no device buffer is allocated. */
+acid_status acid_denoise_loop_graph(const acid_model* m, const acid_loop_cfg* cfg, void* latent,
+                                    const void* text, acid_step_log* log, void* workspace,
+                                    size_t workspace_bytes, acid_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

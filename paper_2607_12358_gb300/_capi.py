@@ -101,6 +101,8 @@ _PROTOS = {
                                     C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
     "acid_denoise_loop": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), _P, _P,
                                     C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
+    "acid_denoise_loop_graph": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), _P, _P,
+                                          C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
 }
 
 _lib = None

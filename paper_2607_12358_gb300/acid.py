@@ -345,14 +345,16 @@ def log_to_dict(lg: A.acid_step_log) -> dict:
 
 
 def acid_denoise_loop(model: DeviceModel, cfg_struct, latent: torch.Tensor, text: torch.Tensor | None = None,
-                      log: bool = True, workspace=None, stream=None) -> list[dict]:
-    """Runs all steps in place on latent (fp32 [C, F, H, W]); returns the step log."""
+                      log: bool = True, workspace=None, stream=None, graph: bool = False) -> list[dict]:
+    """Runs all steps in place on latent (fp32 [C, F, H, W]); returns the step log.
+    ``graph=True`` calls acid_denoise_loop_graph (the whole generation as one CUDA graph)."""
     _need_cuda(latent, text)
     if latent.dtype != torch.float32:
         raise TypeError("latent must be fp32")
     n = cfg_struct.n_steps
     logs = (A.acid_step_log * n)()
     ws, ptr, nbytes = _aligned_ws(model.workspace_size(), latent.device) if workspace is None else workspace
-    check(load().acid_denoise_loop(C.byref(model.struct), C.byref(cfg_struct), latent.data_ptr(), _ptr(text),
-                                   logs if log else None, ptr, nbytes, _stream(stream)))
+    fn = load().acid_denoise_loop_graph if graph else load().acid_denoise_loop
+    check(fn(C.byref(model.struct), C.byref(cfg_struct), latent.data_ptr(), _ptr(text), logs if log else None, ptr,
+             nbytes, _stream(stream)))
     return [log_to_dict(x) for x in logs] if log else []

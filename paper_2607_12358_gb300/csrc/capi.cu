@@ -37,6 +37,8 @@ void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 ProfScope::ProfScope(int kind, double work, cudaStream_t s) : s_(s) {
   std::lock_guard<std::mutex> lk(g_prof_mu);
   if (!g_prof_on) return;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) return;  // not in graphs
   ProfRec r;
   r.kind = kind;
   r.work = work;

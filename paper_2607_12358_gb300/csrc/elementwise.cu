@@ -245,6 +245,89 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
   }
 }
 
+// ------------------------------------------------- fused TEMNI + drift
+// TEMNI_cur = LN(x) (1 + scale) + shift (fp32) and, in the same pass, the
+// sums |TEMNI_cur - TEMNI_prev| and |TEMNI_prev| for the relative-L1 drift.
+// The two TEMNI buffers alternate with the step's parity: cur = tem[step & 1],
+// prev = tem[(step + 1) & 1]; `step` is read from device memory when
+// step_dev is given (graph-launched loops), else step_host is used.  At step
+// 0 there is no previous TEMNI and the sums are zero.  One warp per row
+// (grid-strided), fp64 CTA partials reduced by drift_final_kernel.
+__global__ void __launch_bounds__(kThreads) ln_mod_drift_kernel(const float* __restrict__ x, float* tem0, float* tem1,
+                                                                const int* step_dev, int step_host, int64_t rows, int d,
+                                                                const float* __restrict__ shift,
+                                                                const float* __restrict__ scale, float eps,
+                                                                double2* __restrict__ partials) {
+  const int step = step_dev ? *step_dev : step_host;
+  float* cur = (step & 1) ? tem1 : tem0;
+  const float* prev = (step & 1) ? tem0 : tem1;
+  const bool has_prev = step > 0;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t gw = (int64_t)blockIdx.x * (kThreads / 32) + warp;
+  const int64_t nw = (int64_t)gridDim.x * (kThreads / 32);
+  float num = 0.f, den = 0.f;
+  for (int64_t row = gw; row < rows; row += nw) {
+    const float* xr = x + row * d;
+    float v[kLnMaxV][8];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < kLnMaxV; ++i) {
+      const int c = (i * 32 + lane) * 8;
+      if (c < d) {
+        load8(xr + c, v[i]);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s += v[i][j];
+      }
+    }
+    const float mean = warp_sum_f(s) / d;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < kLnMaxV; ++i) {
+      const int c = (i * 32 + lane) * 8;
+      if (c < d) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float t = v[i][j] - mean;
+          q += t * t;
+        }
+      }
+    }
+    const float rstd = rsqrtf(warp_sum_f(q) / d + eps);
+#pragma unroll
+    for (int i = 0; i < kLnMaxV; ++i) {
+      const int c = (i * 32 + lane) * 8;
+      if (c < d) {
+        float a[8], b[8], o[8];
+        load8(scale + c, a);
+        load8(shift + c, b);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o[j] = fmaf((v[i][j] - mean) * rstd, 1.0f + a[j], b[j]);
+        store8(cur + row * d + c, o);
+        if (has_prev) {
+          float p[8];
+          load8(prev + row * d + c, p);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            num += fabsf(o[j] - p[j]);
+            den += fabsf(p[j]);
+          }
+        }
+      }
+    }
+  }
+  __shared__ double sn[kThreads / 32], sd[kThreads / 32];
+  double dn = warp_sum_d((double)num), dd = warp_sum_d((double)den);
+  if (lane == 0) { sn[warp] = dn; sd[warp] = dd; }
+  __syncthreads();
+  if (warp == 0) {
+    dn = lane < kThreads / 32 ? sn[lane] : 0.0;
+    dd = lane < kThreads / 32 ? sd[lane] : 0.0;
+    dn = warp_sum_d(dn);
+    dd = warp_sum_d(dd);
+    if (lane == 0) partials[blockIdx.x] = make_double2(dn, dd);
+  }
+}
+
 // ---------------------------------------------------------------- GEMV
 template <typename TW>
 __global__ void __launch_bounds__(kThreads) gemv_kernel(const TW* __restrict__ W, const float* __restrict__ b,
@@ -268,12 +351,21 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(const TW* __restrict__ W
   if (lane == 0) y[row] = acc + (b ? b[row] : 0.f);
 }
 
-__global__ void sinusoid_kernel(float* out, double t, int half) {
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= half) return;
+__device__ __forceinline__ void sinusoid_at(float* out, double t, int half, int j) {
   const double f = exp(-log(10000.0) * (double)j / (double)half);
   out[j] = (float)cos(t * f);
   out[half + j] = (float)sin(t * f);
+}
+
+__global__ void sinusoid_kernel(float* out, double t, int half) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j < half) sinusoid_at(out, t, half, j);
+}
+
+// t = 1000 sigma[step] with the step index read from device memory
+__global__ void sinusoid_sig_kernel(float* out, const double* sig, const int* step, int half) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j < half) sinusoid_at(out, 1000.0 * sig[*step], half, j);
 }
 
 __global__ void rope_table_kernel(float2* tbl, int F, int H, int W, int pt, int ph, int pw, double theta) {
@@ -337,6 +429,15 @@ __global__ void unpatchify_euler_kernel(const float* __restrict__ vtok, float* _
 }
 
 __global__ void euler_kernel(float* lat, const float* __restrict__ v, int64_t n, float dsig) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) lat[i] = fmaf(dsig, v[i], lat[i]);
+}
+
+// dsigma = sigma[step + 1] - sigma[step] with the step index read from device memory
+__global__ void euler_sig_kernel(float* lat, const float* __restrict__ v, int64_t n, const double* sig,
+                                 const int* step) {
+  const int i0 = *step;
+  const float dsig = (float)(sig[i0 + 1] - sig[i0]);
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) lat[i] = fmaf(dsig, v[i], lat[i]);
 }
@@ -441,6 +542,22 @@ acid_status ln_mod(int in_dtype, const void* x, int out_dtype, void* y, int64_t 
   return ACID_OK;
 }
 
+acid_status ln_mod_drift(const float* x, float* tem0, float* tem1, const int* step_dev, int step_host, int64_t rows,
+                         int d, const float* shift, const float* scale, float eps, double* d_result, void* workspace,
+                         size_t ws_bytes, cudaStream_t s) {
+  ACID_REQUIRE(d % 8 == 0 && d <= 256 * kLnMaxV, ACID_ERR_UNSUPPORTED, "ln_mod_drift: d must be a multiple of 8, <= 3072");
+  ACID_REQUIRE(ws_bytes >= sizeof(double2) * kDriftMaxBlocks, ACID_ERR_WORKSPACE, "ln_mod_drift: workspace too small");
+  double2* parts = static_cast<double2*>(workspace);
+  const int64_t want = (rows * 32 + kThreads - 1) / kThreads;
+  const int grid = (int)std::min<int64_t>(kDriftMaxBlocks, std::max<int64_t>(1, want));
+  ProfScope prof(PROF_DRIFT, (double)rows * d * 12.0, s);  // read x and prev, write cur (fp32)
+  ln_mod_drift_kernel<<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
+  ACID_CHECK_LAUNCH();
+  drift_final_kernel<<<1, kThreads, 0, s>>>(parts, grid, d_result);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
 acid_status gemv(int w_dtype, const void* W, const float* b, const float* x, float* y, int n_out, int k,
                  bool silu_input, cudaStream_t s) {
   ACID_REQUIRE(k % 8 == 0 && k <= 16384, ACID_ERR_UNSUPPORTED, "gemv: k must be a multiple of 8, <= 16384");
@@ -502,6 +619,20 @@ acid_status unpatchify_euler(const float* vtok, float* v_out, float* latent, int
 
 acid_status euler_update(float* latent, const float* v, int64_t n, float dsigma, cudaStream_t s) {
   euler_kernel<<<grid_for(n), kThreads, 0, s>>>(latent, v, n, dsigma);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status euler_update_sig(float* latent, const float* v, int64_t n, const double* sig, const int* step,
+                             cudaStream_t s) {
+  euler_sig_kernel<<<grid_for(n), kThreads, 0, s>>>(latent, v, n, sig, step);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status timestep_sinusoid_sig(float* out, const double* sig, const int* step, int dim, cudaStream_t s) {
+  const int half = dim / 2;
+  sinusoid_sig_kernel<<<(half + 127) / 128, 128, 0, s>>>(out, sig, step, half);
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }

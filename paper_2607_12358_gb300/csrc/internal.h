@@ -95,6 +95,13 @@ acid_status drift_launch(int dtype, const void* prev, const void* cur, const voi
                          int64_t n, double* d_result /* device double[3]: rel, num, den */,
                          void* workspace, size_t ws_bytes, cudaStream_t s);
 
+// TEMNI = LN(x) (1 + scale) + shift written to tem[step & 1] (fp32), and the
+// relative-L1 drift against tem[(step + 1) & 1] in the same pass; result as
+// drift_launch.  step from step_dev (device) if non-null, else step_host.
+acid_status ln_mod_drift(const float* x, float* tem0, float* tem1, const int* step_dev, int step_host, int64_t rows,
+                         int d, const float* shift, const float* scale, float eps, double* d_result, void* workspace,
+                         size_t ws_bytes, cudaStream_t s);
+
 // out = a + b elementwise, one dtype, 16-byte vectors
 acid_status add_same(int dtype, const void* a, const void* b, void* out, int64_t n, cudaStream_t s);
 
@@ -108,5 +115,10 @@ acid_status patchify(const float* latent, int out_dtype, void* tokens, int C, in
 acid_status unpatchify_euler(const float* vtok, float* v_out, float* latent, int C, int F, int H,
                              int W, int pt, int ph, int pw, float dsigma, cudaStream_t s);
 acid_status euler_update(float* latent, const float* v, int64_t n, float dsigma, cudaStream_t s);
+// Variants that read the step index from device memory (graph-launched loops):
+// t = 1000 sig[*step]; dsigma = sig[*step + 1] - sig[*step].
+acid_status euler_update_sig(float* latent, const float* v, int64_t n, const double* sig, const int* step,
+                             cudaStream_t s);
+acid_status timestep_sinusoid_sig(float* out, const double* sig, const int* step, int dim, cudaStream_t s);
 
 }  // namespace acid

@@ -39,7 +39,25 @@ struct LoopWs {
   uint8_t* drift_ws;
   float2* rope;
   uint8_t* block_base;
+  // device-side loop state for graph-launched generations
+  struct DevLoop* dev;      // controller state and configuration
+  double* sig;              // [kMaxGraphSteps + 1] noise levels
+  int8_t* forced;           // [kMaxGraphSteps]
+  acid_step_log* dlog;      // [kMaxGraphSteps]
   size_t bytes;
+};
+
+constexpr int kMaxGraphSteps = 1024;
+
+// Algorithm 1's state and inputs as the device controller sees them.
+struct DevLoop {
+  int step;  // first member: the kernels read the step index through &dev->step
+  int have_prev, have_cache, have_rate;
+  int n_steps, warmup, method, force_last, use_forced;
+  int compute;
+  double sigma_acc, s_prev, k_rate;
+  double tau_low, tau_high, delta;
+  double latent_n;
 };
 
 struct Shape {
@@ -102,6 +120,10 @@ LoopWs loop_layout(const acid_model& m, void* base) {
   size_t blk = block_ws_layout(desc_for(m, 0), nullptr).bytes;
   blk = std::max(blk, block_ws_layout(desc_for(m, total_blocks(m) - 1), nullptr).bytes);
   w.block_base = b.take<uint8_t>(blk);
+  w.dev = b.take<DevLoop>(1);
+  w.sig = b.take<double>(kMaxGraphSteps + 1);
+  w.forced = b.take<int8_t>(kMaxGraphSteps);
+  w.dlog = b.take<acid_step_log>(kMaxGraphSteps);
   w.bytes = b.off + 1024;
   return w;
 }
@@ -329,14 +351,13 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
   bool compute = true;
   if (cfg->method == ACID_METHOD_TEACACHE) {
     // s_t: rel_l1 of block 0's modulated input between consecutive steps
-    const int cur = i & 1, prv = cur ^ 1;
+    // TEMNI_i = block 0's modulated input, written to temni[i & 1], and its
+    // drift against TEMNI_{i-1} in temni[(i + 1) & 1], in one pass
     ACID_TRY(gemv(dt, m->blocks[0].mod.w, m->blocks[0].mod.b, w.temb, w.mod0, 2 * sh.d, sh.d, true, s));
-    ACID_TRY(ln_mod(ACID_FP32, w.h_in, ACID_FP32, w.temni[cur], sh.N, sh.d, w.mod0, w.mod0 + sh.d, nullptr, nullptr,
-                    0, m->block.ln_eps, s));
+    ACID_TRY(ln_mod_drift(w.h_in, w.temni[0], w.temni[1], nullptr, i, sh.N, sh.d, w.mod0, w.mod0 + sh.d,
+                          m->block.ln_eps, w.dres, w.drift_ws, drift_workspace_bytes(0), s));
     if (!warm) {
       ACID_REQUIRE(i > 0, ACID_ERR_INVALID_ARG, "TeaCache needs at least one warmup step");
-      ACID_TRY(drift_launch(ACID_FP32, w.temni[prv], w.temni[cur], nullptr, nullptr, sh.N * sh.d, w.dres,
-                            w.drift_ws, drift_workspace_bytes(0), s));
       double h[3];
       ACID_TRY(read_results(h, w.dres, 3, s));
       compute = controller_step(*st, *cfg, h[0], forced, &lg);
@@ -410,4 +431,280 @@ extern "C" acid_status acid_denoise_loop(const acid_model* m, const acid_loop_cf
   for (int i = 0; i < cfg->n_steps; ++i)
     ACID_TRY(acid_denoise_step(m, cfg, &st, latent, log ? log + i : nullptr, workspace, workspace_bytes, stream));
   return ACID_OK;
+}
+
+// ===========================================================================
+// The whole generation as one CUDA graph: a WHILE node whose body is one
+// sampler step.  The drift signal, Algorithm 1's decision and the step index
+// live in device memory; the decision selects the IF (compute) or ELSE
+// (reuse) body of a conditional node, so no step waits for the host.
+// ===========================================================================
+
+namespace acid {
+namespace {
+
+__device__ double dev_ratio_or_inf(double num, double den) {
+  if (den == 0.0) return num == 0.0 ? 0.0 : INFINITY;
+  return num / den;
+}
+
+// Algorithm 1 on the device (one thread): same arithmetic as controller_step.
+// dres: TeaCache {rel, num, den}; EasyCache {., sum|x - x_prev|, .,
+// ., ., sum|v_prev|}.
+__global__ void controller_kernel(DevLoop* st, const double* dres, const double* sig, const int8_t* forced,
+                                  acid_step_log* log, cudaGraphConditionalHandle h_compute) {
+  const int i = st->step;
+  const bool warm = i < st->warmup;
+  int f = st->use_forced ? forced[i] : -1;
+  if (f < 0 && st->force_last && i == st->n_steps - 1) f = 1;
+  acid_step_log lg;
+  lg.step = i;
+  lg.warmup = warm;
+  lg.forced = 0;
+  lg.t = 1000.0 * sig[i];
+  lg.signal = lg.dsignal = lg.tau = lg.sigma = NAN;
+  lg.ms = NAN;
+  bool compute = true;
+  if (!warm) {
+    const double s = st->method == ACID_METHOD_TEACACHE
+                         ? dres[0]
+                         : dev_ratio_or_inf(st->k_rate * (dres[1] / st->latent_n), dres[5] / st->latent_n);
+    st->sigma_acc += s;
+    double tau, ds = NAN;
+    if (st->have_prev) {
+      ds = fabs(s - st->s_prev);
+      tau = ds <= st->delta ? st->tau_high : st->tau_low;
+    } else {
+      tau = st->tau_low;
+    }
+    const double seen = st->sigma_acc;
+    bool skip = seen <= tau;
+    if (f >= 0) skip = f == 0;
+    if (!skip) st->sigma_acc = 0.0;
+    st->s_prev = s;
+    st->have_prev = 1;
+    compute = !skip;
+    lg.signal = s;
+    lg.dsignal = ds;
+    lg.tau = tau;
+    lg.sigma = seen;
+    lg.forced = f >= 0;
+  }
+  if (!st->have_cache) compute = true;
+  if (compute) st->have_cache = 1;
+  st->compute = compute;
+  lg.computed = compute;
+  log[i] = lg;
+  cudaGraphSetConditional(h_compute, compute ? 1u : 0u);
+}
+
+// EasyCache k = mean|v_c - v_{c-1}| / mean|x_c - x_{c-1}| after a computed step i > 0.
+__global__ void easycache_rate_kernel(DevLoop* st, const double* dres) {
+  if (st->step == 0) return;
+  st->k_rate = dev_ratio_or_inf(dres[1] / st->latent_n, dres[4] / st->latent_n);
+  st->have_rate = 1;
+}
+
+__global__ void advance_kernel(DevLoop* st, cudaGraphConditionalHandle h_loop) {
+  st->step += 1;
+  cudaGraphSetConditional(h_loop, st->step < st->n_steps ? 1u : 0u);
+}
+
+acid_status add_conditional(cudaStream_t s, cudaGraphConditionalHandle h, cudaGraphConditionalNodeType type,
+                            unsigned size, cudaGraph_t* bodies) {
+  cudaStreamCaptureStatus status;
+  cudaGraph_t g;
+  const cudaGraphNode_t* deps = nullptr;
+  size_t ndeps = 0;
+  ACID_CUDA(cudaStreamGetCaptureInfo(s, &status, nullptr, &g, &deps, nullptr, &ndeps));
+  ACID_REQUIRE(status == cudaStreamCaptureStatusActive, ACID_ERR_CUDA, "graph: stream is not capturing");
+  cudaGraphNodeParams p = {};
+  p.type = cudaGraphNodeTypeConditional;
+  p.conditional.handle = h;
+  p.conditional.type = type;
+  p.conditional.size = size;
+  cudaGraphNode_t node;
+  ACID_CUDA(cudaGraphAddNode(&node, g, deps, nullptr, ndeps, &p));
+  for (unsigned k = 0; k < size; ++k) bodies[k] = p.conditional.phGraph_out[k];
+  ACID_CUDA(cudaStreamUpdateCaptureDependencies(s, &node, nullptr, 1, cudaStreamSetCaptureDependencies));
+  return ACID_OK;
+}
+
+struct GraphCapture {
+  cudaStream_t main = nullptr, side = nullptr;
+  ~GraphCapture() {
+    if (main) cudaStreamDestroy(main);
+    if (side) cudaStreamDestroy(side);
+  }
+};
+
+// Records one step into `body` (captured on gc.main; conditional bodies on gc.side).
+acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& w, float* latent, GraphCapture& gc,
+                         cudaGraph_t body, cudaGraphConditionalHandle h_loop) {
+  const Shape sh = shape_of(m);
+  const int dt = m.block.dtype;
+  cudaStream_t s = gc.main, s2 = gc.side;
+  const int* step = &w.dev->step;
+  const int64_t vrow0 = m.block.kind == ACID_BLOCK_WAN ? 0 : sh.L;
+  void* x_video = w.xbuf + vrow0 * sh.d * es(dt);
+  cudaGraphConditionalHandle h_compute;
+  ACID_CUDA(cudaGraphConditionalHandleCreate(&h_compute, body, 0, 0));
+
+  ACID_CUDA(cudaStreamBeginCaptureToGraph(s, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  // ---- step inputs: temb, patch embedding
+  ACID_TRY(timestep_sinusoid_sig(w.sinus, w.sig, step, m.time_freq_dim, s));
+  ACID_TRY(gemv(dt, m.time1.w, m.time1.b, w.sinus, w.temb_h, sh.d, m.time_freq_dim, false, s));
+  ACID_TRY(gemv(dt, m.time2.w, m.time2.b, w.temb_h, w.temb, sh.d, sh.d, true, s));
+  ACID_TRY(patchify(latent, ACID_FP32, w.tokens, m.latent_c, m.latent_f, m.latent_h, m.latent_w, m.pt, m.ph, m.pw, s));
+  {
+    Epilogue e;
+    e.bias = m.patch.b;
+    e.out_fp32 = true;
+    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m.patch.w, sh.d, w.h_in, sh.d, e, s));
+  }
+  // ---- signal and decision
+  float* v = w.v[0];
+  float* v_prev = w.v[1];
+  if (cfg.method == ACID_METHOD_TEACACHE) {
+    ACID_TRY(gemv(dt, m.blocks[0].mod.w, m.blocks[0].mod.b, w.temb, w.mod0, 2 * sh.d, sh.d, true, s));
+    ACID_TRY(ln_mod_drift(w.h_in, w.temni[0], w.temni[1], step, 0, sh.N, sh.d, w.mod0, w.mod0 + sh.d, m.block.ln_eps,
+                          w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+  } else {
+    ACID_TRY(drift_launch(ACID_FP32, w.x_prev, latent, nullptr, nullptr, sh.latent, w.dres, w.drift_ws,
+                          drift_workspace_bytes(0), s));
+    ACID_TRY(drift_launch(ACID_FP32, v_prev, v_prev, nullptr, nullptr, sh.latent, w.dres + 3, w.drift_ws,
+                          drift_workspace_bytes(0), s));
+  }
+  controller_kernel<<<1, 1, 0, s>>>(w.dev, w.dres, w.sig, w.forced, w.dlog, h_compute);
+  ACID_CHECK_LAUNCH();
+  cudaGraph_t br[2];
+  ACID_TRY(add_conditional(s, h_compute, cudaGraphCondTypeIf, 2, br));
+
+  // ---- compute body: the model
+  ACID_CUDA(cudaStreamBeginCaptureToGraph(s2, br[0], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s2));
+  ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s2));
+  ACID_TRY(run_blocks(m, w, s2));
+  if (cfg.method == ACID_METHOD_TEACACHE) {
+    ACID_TRY(add_mixed(dt, x_video, ACID_FP32, w.h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s2));
+  } else {
+    ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s2));
+    ACID_TRY(drift_launch(ACID_FP32, v_prev, v, nullptr, nullptr, sh.latent, w.dres, w.drift_ws,
+                          drift_workspace_bytes(0), s2));
+    ACID_TRY(drift_launch(ACID_FP32, w.x_prev, latent, nullptr, nullptr, sh.latent, w.dres + 3, w.drift_ws,
+                          drift_workspace_bytes(0), s2));
+    easycache_rate_kernel<<<1, 1, 0, s2>>>(w.dev, w.dres);
+    ACID_CHECK_LAUNCH();
+    ACID_TRY(add_mixed(ACID_FP32, v, ACID_FP32, latent, ACID_FP32, w.offset, sh.latent, -1.0f, s2));
+  }
+  cudaGraph_t tmp;
+  ACID_CUDA(cudaStreamEndCapture(s2, &tmp));
+  // ---- reuse body: cached residual / offset
+  ACID_CUDA(cudaStreamBeginCaptureToGraph(s2, br[1], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  if (cfg.method == ACID_METHOD_TEACACHE)
+    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s2));
+  else
+    ACID_TRY(add_mixed(ACID_FP32, latent, ACID_FP32, w.offset, ACID_FP32, v, sh.latent, 1.0f, s2));
+  ACID_CUDA(cudaStreamEndCapture(s2, &tmp));
+
+  // ---- output: velocity and the Euler update, then the next step
+  if (cfg.method == ACID_METHOD_TEACACHE) {
+    ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s));
+  } else {
+    ACID_CUDA(cudaMemcpyAsync(w.x_prev, latent, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
+    ACID_CUDA(cudaMemcpyAsync(v_prev, v, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
+  }
+  ACID_TRY(euler_update_sig(latent, v, sh.latent, w.sig, step, s));
+  advance_kernel<<<1, 1, 0, s>>>(w.dev, h_loop);
+  ACID_CHECK_LAUNCH();
+  ACID_CUDA(cudaStreamEndCapture(s, &tmp));
+  return ACID_OK;
+}
+
+}  // namespace
+}  // namespace acid
+
+extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_loop_cfg* cfg, void* latent_v,
+                                               const void* text, acid_step_log* log, void* workspace,
+                                               size_t workspace_bytes, acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m && cfg && latent_v, ACID_ERR_INVALID_ARG, "acid_denoise_loop_graph: null argument");
+  ACID_TRY(validate_cfg(*cfg));
+  ACID_REQUIRE(cfg->n_steps <= kMaxGraphSteps, ACID_ERR_UNSUPPORTED,
+               "acid_denoise_loop_graph: at most " + std::to_string(kMaxGraphSteps) + " steps");
+  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_denoise_loop_graph: latent must be 16-byte aligned");
+  acid_loop_state st;
+  ACID_TRY(acid_loop_begin(m, cfg, text, &st, workspace, workspace_bytes, stream));
+  LoopWs w = loop_layout(*m, workspace);
+  cudaStream_t s = (cudaStream_t)stream;
+  const Shape sh = shape_of(*m);
+  // device state, noise levels and forced decisions
+  DevLoop d = {};
+  d.n_steps = cfg->n_steps;
+  d.warmup = cfg->warmup;
+  d.method = cfg->method;
+  d.force_last = cfg->force_last;
+  d.use_forced = cfg->forced != nullptr;
+  d.tau_low = cfg->tau_low;
+  d.tau_high = cfg->tau_high;
+  d.delta = cfg->delta;
+  d.latent_n = (double)sh.latent;
+  double sig[kMaxGraphSteps + 1];
+  for (int i = 0; i <= cfg->n_steps; ++i) sig[i] = sigma_at(*cfg, i);
+  ACID_CUDA(cudaMemcpyAsync(w.dev, &d, sizeof(d), cudaMemcpyHostToDevice, s));
+  ACID_CUDA(cudaMemcpyAsync(w.sig, sig, sizeof(double) * (cfg->n_steps + 1), cudaMemcpyHostToDevice, s));
+  if (cfg->forced)
+    ACID_CUDA(cudaMemcpyAsync(w.forced, cfg->forced, cfg->n_steps, cudaMemcpyHostToDevice, s));
+  ACID_CUDA(cudaStreamSynchronize(s));  // host sources above are stack memory
+
+  GraphCapture gc;
+  ACID_CUDA(cudaStreamCreateWithFlags(&gc.main, cudaStreamNonBlocking));
+  ACID_CUDA(cudaStreamCreateWithFlags(&gc.side, cudaStreamNonBlocking));
+  cudaGraph_t g = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  acid_status rc = ACID_OK;
+  do {
+    if (cudaGraphCreate(&g, 0) != cudaSuccess) { rc = ACID_ERR_CUDA; set_error("cudaGraphCreate failed"); break; }
+    cudaGraphConditionalHandle h_loop;
+    if (cudaGraphConditionalHandleCreate(&h_loop, g, 1, cudaGraphCondAssignDefault) != cudaSuccess) {
+      rc = ACID_ERR_CUDA;
+      set_error("cudaGraphConditionalHandleCreate failed");
+      break;
+    }
+    cudaGraphNodeParams p = {};
+    p.type = cudaGraphNodeTypeConditional;
+    p.conditional.handle = h_loop;
+    p.conditional.type = cudaGraphCondTypeWhile;
+    p.conditional.size = 1;
+    cudaGraphNode_t node;
+    if (cudaGraphAddNode(&node, g, nullptr, nullptr, 0, &p) != cudaSuccess) {
+      rc = ACID_ERR_CUDA;
+      set_error("cudaGraphAddNode (while) failed");
+      break;
+    }
+    rc = capture_step(*m, *cfg, w, static_cast<float*>(latent_v), gc, p.conditional.phGraph_out[0], h_loop);
+    if (rc != ACID_OK) {
+      cudaGraph_t junk;
+      cudaStreamEndCapture(gc.side, &junk);
+      cudaStreamEndCapture(gc.main, &junk);
+      break;
+    }
+    cudaError_t e = cudaGraphInstantiate(&exec, g, 0);
+    if (e != cudaSuccess) {
+      rc = ACID_ERR_CUDA;
+      set_error(std::string("cudaGraphInstantiate: ") + cudaGetErrorString(e));
+      break;
+    }
+    e = cudaGraphLaunch(exec, s);
+    if (e == cudaSuccess && log)
+      e = cudaMemcpyAsync(log, w.dlog, sizeof(acid_step_log) * cfg->n_steps, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) {
+      rc = ACID_ERR_CUDA;
+      set_error(std::string("graph launch: ") + cudaGetErrorString(e));
+    }
+  } while (false);
+  if (exec) cudaGraphExecDestroy(exec);
+  if (g) cudaGraphDestroy(g);
+  return rc;
 }
