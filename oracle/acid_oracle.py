@@ -97,6 +97,29 @@ def easycache_reuse(x_t, x_c, v_c) -> np.ndarray:
     return np.asarray(x_t, F64) + (np.asarray(v_c, F64) - np.asarray(x_c, F64))
 
 
+def dicache_gamma(p_t, p_c1, p_c2) -> float:
+    """Probe-trajectory ratio |P_t - P_c1|_1 / |P_c1 - P_c2|_1 (0 when the
+    denominator is 0, i.e. fewer than two distinct computed steps)."""
+    den = float(np.abs(np.asarray(p_c1, F64) - np.asarray(p_c2, F64)).sum())
+    if den == 0.0:
+        return 0.0
+    return float(np.abs(np.asarray(p_t, F64) - np.asarray(p_c1, F64)).sum()) / den
+
+
+def dicache_reuse(p_t, p_c1, p_c2, d_c1, d_c2) -> np.ndarray:
+    """DiCache reconstruction on a skipped step (Sec. 2, "DiCache": the deep
+    output is estimated from the probe features' trajectory over recent
+    steps).  Reading: with D = H_out - P the deep part beyond the probe at
+    the last two computed steps c1 (latest) and c2,
+        H_out_t = P_t + D_c1 + gamma (D_c1 - D_c2),
+        gamma = |P_t - P_c1|_1 / |P_c1 - P_c2|_1,
+    i.e. the deep part moves along its last computed direction in proportion
+    to how far the probe has moved since."""
+    g = dicache_gamma(p_t, p_c1, p_c2)
+    d1 = np.asarray(d_c1, F64)
+    return np.asarray(p_t, F64) + d1 + g * (d1 - np.asarray(d_c2, F64))
+
+
 # =============================================================================
 # Adaptive threshold controller (Sec. 3.3, Algorithm 1)
 # =============================================================================
@@ -533,34 +556,44 @@ def text_context(cfg, w, text):
     return np.asarray(text, F64)
 
 
+def stack_state(cfg, h_in, ctx) -> np.ndarray:
+    """Hidden state entering the block stack: the video tokens (Wan) or
+    [text ; video] (joint models)."""
+    if cfg.kind == "wan":
+        return np.asarray(h_in, F64)
+    return np.concatenate([np.asarray(ctx, F64), np.asarray(h_in, F64)], axis=0)
+
+
+def state_video(cfg, state, ctx) -> np.ndarray:
+    return state if cfg.kind == "wan" else state[ctx.shape[0]:]
+
+
+def run_block_range(cfg, w, state, mods, ctx, b0, b1) -> np.ndarray:
+    """Blocks b0 <= i < b1 applied to a stack state (see stack_state)."""
+    grid = cfg.grid
+    H = cfg.heads
+    x = np.asarray(state, F64)
+    L = 0 if cfg.kind == "wan" else ctx.shape[0]
+    for i in range(b0, b1):
+        wb, m = w["blocks"][i], mods[i]
+        if cfg.kind == "wan":
+            x = wan_block(x, m, wb, grid, H, ctx=ctx, eps=cfg.ln_eps, theta=cfg.rope_theta)
+        elif cfg.kind == "cog":
+            x = cog_block(x, m, wb, grid, H, L, eps=cfg.ln_eps, theta=cfg.rope_theta)
+        elif i < cfg.n_blocks:  # hv dual-stream
+            mv, mt = m
+            xt, xv = hv_dual_block(x[:L], x[L:], mt, mv, wb, grid, H, eps=cfg.ln_eps, theta=cfg.rope_theta)
+            x = np.concatenate([xt, xv], axis=0)
+        else:  # hv single-stream
+            x = hv_single_block(x, m, wb, grid, H, L, eps=cfg.ln_eps, theta=cfg.rope_theta)
+    return x
+
+
 def block_stack(cfg, w, h_in, mods, ctx) -> np.ndarray:
     """Run every block on the video tokens h_in (and the text stream for joint
     models); returns the video tokens after the last block."""
-    grid = cfg.grid
-    H = cfg.heads
-    if cfg.kind == "wan":
-        x = h_in
-        for wb, m in zip(w["blocks"], mods):
-            x = wan_block(x, m, wb, grid, H, ctx=ctx, eps=cfg.ln_eps, theta=cfg.rope_theta)
-        return x
-    if cfg.kind == "cog":
-        L = ctx.shape[0]
-        x = np.concatenate([ctx, h_in], axis=0)
-        for wb, m in zip(w["blocks"], mods):
-            x = cog_block(x, m, wb, grid, H, L, eps=cfg.ln_eps, theta=cfg.rope_theta)
-        return x[L:]
-    if cfg.kind == "hv":
-        L = ctx.shape[0]
-        xt, xv = ctx, h_in
-        nd = cfg.n_blocks
-        for wb, m in zip(w["blocks"][:nd], mods[:nd]):
-            mv, mt = m
-            xt, xv = hv_dual_block(xt, xv, mt, mv, wb, grid, H, eps=cfg.ln_eps, theta=cfg.rope_theta)
-        x = np.concatenate([xt, xv], axis=0)
-        for wb, m in zip(w["blocks"][nd:], mods[nd:]):
-            x = hv_single_block(x, m, wb, grid, H, L, eps=cfg.ln_eps, theta=cfg.rope_theta)
-        return x[L:]
-    raise ValueError(cfg.kind)
+    state = run_block_range(cfg, w, stack_state(cfg, h_in, ctx), mods, ctx, 0, len(w["blocks"]))
+    return state_video(cfg, state, ctx)
 
 
 def final_layer(cfg, w, h_out, final_mod) -> np.ndarray:
@@ -588,9 +621,11 @@ class LoopResult:
 
 
 def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None, delta=None,
-                 warmup=None, method=None, forced=None, force_last=False, shift=1.0) -> LoopResult:
+                 warmup=None, method=None, forced=None, force_last=False, shift=1.0,
+                 probe_blocks=1) -> LoopResult:
     """The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler
-    flow-matching sampler, with TeaCache or EasyCache as the base method M.
+    flow-matching sampler, with TeaCache, EasyCache or DiCache as the base
+    method M.
 
     TeaCache (Sec. 2): s_t = rel_l1(TEMNI_{t-1}, TEMNI_t) between consecutive
     steps (computed or not); M.update stores R = H_out - H_in of the block
@@ -598,6 +633,11 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
     EasyCache (Sec. 2): s_t = k * mean|x_t - x_{t-1}| / mean|v_{t-1}|;
     M.update refreshes k and the offset v_c - x_c; M.reuse gives
     v_t = x_t + (v_c - x_c).
+
+    DiCache (Sec. 2): the first ``probe_blocks`` blocks run on every step;
+    s_t = rel_l1(P_{t-1}, P_t) of the probe features; M.update keeps the probe
+    features and deep parts D = H_out - P of the last two computed steps;
+    M.reuse is dicache_reuse.
 
     ``forced``: optional per-step list of None/True/False; True or False
     replaces the controller's decision at that step (compute / skip).
@@ -618,6 +658,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
     x_prev = v_prev = None
     x_c = v_c = None
     k_rate = None
+    probe_prev = p_c1 = p_c2 = d_c1 = d_c2 = None
     for i in range(n_steps):
         t = 1000.0 * sig[i]
         rec = StepRecord(step=i, warmup=i < warmup)
@@ -660,6 +701,31 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
             else:
                 v = easycache_reuse(x, x_c, v_c)
             x_prev, v_prev = x, v
+        elif method == "dicache":
+            # probe: the first probe_blocks blocks, run on every step
+            state = run_block_range(cfg, w, stack_state(cfg, si.h_in, ctx), si.mods, ctx, 0, probe_blocks)
+            probe = state_video(cfg, state, ctx)
+            if i < warmup:
+                compute = True
+            else:
+                s = rel_l1(probe_prev, probe)
+                skip, tau, sg, ds = ctl.step(s, forced=f)
+                rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
+                compute = not skip
+                rec.forced = f is not None
+            probe_prev = probe
+            if compute:
+                state = run_block_range(cfg, w, state, si.mods, ctx, probe_blocks, len(w["blocks"]))
+                h_out = state_video(cfg, state, ctx)
+                d_new = h_out - probe
+                if p_c1 is None:
+                    p_c2, d_c2 = probe, d_new
+                else:
+                    p_c2, d_c2 = p_c1, d_c1
+                p_c1, d_c1 = probe, d_new
+            else:
+                h_out = dicache_reuse(probe, p_c1, p_c2, d_c1, d_c2)
+            v = final_layer(cfg, w, h_out, si.final_mod)
         else:
             raise ValueError(method)
         rec.computed = compute

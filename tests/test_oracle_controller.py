@@ -212,3 +212,47 @@ def test_easycache_loop_runs_and_warms_up_two_steps():
     r = O.denoise_loop(cfg, w, S.latent(cfg, 1), None)
     assert r.computed[:2] == [True, True]
     assert all(np.isfinite(rec.signal) for rec in r.records[2:])
+
+
+# ---------------------------------------------------------------------------
+# DiCache reading (Sec. 2, "DiCache")
+# ---------------------------------------------------------------------------
+
+def test_dicache_reuse_exact_on_straight_trajectory():
+    """Probe and deep part moving along one straight line with proportional
+    steps: the trajectory extrapolation is exact."""
+    rng = np.random.default_rng(21)
+    p2, dp = rng.normal(size=(5, 7)), rng.normal(size=(5, 7))
+    d2, dd = rng.normal(size=(5, 7)), rng.normal(size=(5, 7))
+    p1, d1 = p2 + dp, d2 + dd
+    for a in (0.5, 1.0, 2.5):
+        pt = p1 + a * dp
+        assert O.dicache_gamma(pt, p1, p2) == pytest.approx(a)
+        np.testing.assert_allclose(O.dicache_reuse(pt, p1, p2, d1, d2), pt + d1 + a * dd, atol=1e-12)
+
+
+def test_dicache_single_cached_step_reuses_deep_part():
+    rng = np.random.default_rng(22)
+    p, d, pt = rng.normal(size=(3, 4)), rng.normal(size=(3, 4)), rng.normal(size=(3, 4))
+    assert O.dicache_gamma(pt, p, p) == 0.0
+    np.testing.assert_allclose(O.dicache_reuse(pt, p, p, d, d), pt + d, atol=0)
+
+
+def test_dicache_full_depth_probe_is_uncached():
+    """A probe as deep as the whole stack leaves no deep part (D = 0), so every
+    reuse reproduces the model output exactly, whatever the decisions."""
+    cfg = S.get_config("toy", steps=6)
+    w = S.model_weights(cfg, 8)
+    lat = S.latent(cfg, 8)
+    r = O.denoise_loop(cfg, w, lat, None, method="dicache", probe_blocks=cfg.n_blocks, tau_low=1e9, tau_high=1e9)
+    assert r.computed == [True] + [False] * (cfg.steps - 1)
+    np.testing.assert_allclose(r.latent, _plain_sampler(cfg, w, lat, cfg.steps), atol=1e-12)
+
+
+def test_dicache_negative_threshold_is_uncached():
+    cfg = S.get_config("toy", steps=5)
+    w = S.model_weights(cfg, 9)
+    lat = S.latent(cfg, 9)
+    r = O.denoise_loop(cfg, w, lat, None, method="dicache", tau_low=-1.0, tau_high=-1.0)
+    assert all(r.computed)
+    np.testing.assert_allclose(r.latent, _plain_sampler(cfg, w, lat, cfg.steps), atol=1e-12)
