@@ -53,7 +53,11 @@ typedef enum {
   ACID_BLOCK_HV_SINGLE = 3  /* joint single stream, parallel attention + MLP */
 } acid_block_kind;
 
-typedef enum { ACID_METHOD_TEACACHE = 0, ACID_METHOD_EASYCACHE = 1 } acid_method;
+typedef enum {
+  ACID_METHOD_TEACACHE = 0,   /* Sec. 2 "TeaCache": drift of block 0's modulated input */
+  ACID_METHOD_EASYCACHE = 1,  /* Sec. 2 "EasyCache": k * input change / output magnitude */
+  ACID_METHOD_DICACHE = 2     /* Sec. 2 "DiCache": drift of shallow probe-block features */
+} acid_method;
 
 /* Message of the last failed call on this thread ("" if none). */
 const char* acid_last_error(void);
@@ -289,6 +293,7 @@ typedef struct {
   double delta;              /* stability bound on |s_t - s_prev| */
   double shift;              /* sigma shift s (1 = none) */
   const int8_t* forced;      /* host [n_steps] or NULL: -1 controller, 0 reuse, 1 compute */
+  int32_t probe_blocks;      /* DiCache: blocks run on every step as the probe (>= 1) */
 } acid_loop_cfg;
 
 typedef struct {
@@ -328,8 +333,12 @@ acid_status acid_loop_begin(const acid_model* m, const acid_loop_cfg* cfg, const
  *   t = 1000 sigma_i; temb; patch embedding H_in of the latent;
  *   on non-warmup steps s_t (TeaCache: rel_l1 of block 0's modulated input
  *   between consecutive steps; EasyCache: k mean|x_t - x_{t-1}| /
- *   mean|v_{t-1}|), Sigma += s_t, tau by |s_t - s_prev| <= delta, reuse iff
- *   Sigma <= tau, else run all blocks and reset Sigma;
+ *   mean|v_{t-1}|; DiCache: rel_l1 of the probe blocks' output P between
+ *   consecutive steps), Sigma += s_t, tau by |s_t - s_prev| <= delta, reuse
+ *   iff Sigma <= tau, else run all (remaining) blocks and reset Sigma.
+ *   DiCache reuse (a reading; the paper describes it only in words):
+ *   H_out = P_t + D_1 + g (D_1 - D_2), D = H_out - P at the last two computed
+ *   steps, g = |P_t - P_1|_1 / |P_1 - P_2|_1 (0 when P_1 = P_2);
  *   final layer, x_{i+1} = x_i + (sigma_{i+1} - sigma_i) v.
  *   latent    device fp32 [C, F, H, W], updated in place.
  *   log       host, one entry written, or NULL.

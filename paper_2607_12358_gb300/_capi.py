@@ -14,7 +14,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libacid_gb
 ACID_OK, ACID_ERR_INVALID_ARG, ACID_ERR_UNSUPPORTED, ACID_ERR_WORKSPACE, ACID_ERR_CUDA, ACID_ERR_TIMEOUT = range(6)
 ACID_BF16, ACID_FP32 = 0, 1
 ACID_BLOCK_WAN, ACID_BLOCK_COG, ACID_BLOCK_HV_DUAL, ACID_BLOCK_HV_SINGLE = range(4)
-ACID_METHOD_TEACACHE, ACID_METHOD_EASYCACHE = 0, 1
+ACID_METHOD_TEACACHE, ACID_METHOD_EASYCACHE, ACID_METHOD_DICACHE = 0, 1, 2
 ACID_EPI_BIAS, ACID_EPI_GELU, ACID_EPI_GATED_RES, ACID_EPI_RES = 0, 1, 3, 4
 
 STATUS_NAMES = {0: "ACID_OK", 1: "ACID_ERR_INVALID_ARG", 2: "ACID_ERR_UNSUPPORTED", 3: "ACID_ERR_WORKSPACE",
@@ -55,7 +55,7 @@ class acid_model(C.Structure):
 class acid_loop_cfg(C.Structure):
     _fields_ = [("n_steps", C.c_int32), ("warmup", C.c_int32), ("method", C.c_int32), ("force_last", C.c_int32),
                 ("tau_low", C.c_double), ("tau_high", C.c_double), ("delta", C.c_double), ("shift", C.c_double),
-                ("forced", C.POINTER(C.c_int8))]
+                ("forced", C.POINTER(C.c_int8)), ("probe_blocks", C.c_int32)]
 
 
 class acid_step_log(C.Structure):

@@ -292,14 +292,18 @@ class DeviceModel:
         return b.value
 
 
+_METHOD = {"teacache": A.ACID_METHOD_TEACACHE, "easycache": A.ACID_METHOD_EASYCACHE, "dicache": A.ACID_METHOD_DICACHE}
+
+
 def loop_cfg(cfg, n_steps=None, tau_low=None, tau_high=None, delta=None, warmup=None, method=None,
-             force_last=False, shift=1.0, forced=None):
+             force_last=False, shift=1.0, forced=None, probe_blocks=1):
     """acid_loop_cfg from a workload config; returns (struct, keepalive)."""
     method = cfg.method if method is None else method
     c = A.acid_loop_cfg()
     c.n_steps = cfg.steps if n_steps is None else n_steps
-    c.warmup = cfg.warmup if warmup is None else warmup
-    c.method = A.ACID_METHOD_EASYCACHE if method == "easycache" else A.ACID_METHOD_TEACACHE
+    c.warmup = (2 if method == "easycache" else 1) if warmup is None else warmup
+    c.method = _METHOD[method]
+    c.probe_blocks = probe_blocks
     c.force_last = int(bool(force_last))
     c.tau_low = cfg.tau_low if tau_low is None else tau_low
     c.tau_high = cfg.tau_high if tau_high is None else tau_high

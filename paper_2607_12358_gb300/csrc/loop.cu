@@ -35,6 +35,12 @@ struct LoopWs {
   float* v[2];      // latent-sized velocity, current / previous (EasyCache)
   float* x_prev;    // latent-sized previous input (EasyCache)
   float* offset;    // latent-sized v_c - x_c (EasyCache)
+  // DiCache: probe features of the current / previous step are temni[], the
+  // deep part D_1 = H_out - P of the last computed step is resid
+  float* dc_p1;     // [N, d] probe features of the last computed step
+  float* dc_p2;     // [N, d] probe features of the computed step before
+  float* dc_d2;     // [N, d] deep part of the computed step before
+  int* dc_count;    // computed steps cached (0, 1, 2)
   double* dres;     // [8] device drift results
   uint8_t* drift_ws;
   float2* rope;
@@ -112,6 +118,10 @@ LoopWs loop_layout(const acid_model& m, void* base) {
   w.v[1] = b.take<float>(s.latent);
   w.x_prev = b.take<float>(s.latent);
   w.offset = b.take<float>(s.latent);
+  w.dc_p1 = b.take<float>(s.N * s.d);
+  w.dc_p2 = b.take<float>(s.N * s.d);
+  w.dc_d2 = b.take<float>(s.N * s.d);
+  w.dc_count = b.take<int>(1);
   w.dres = b.take<double>(8);
   w.drift_ws = b.take<uint8_t>(drift_workspace_bytes(0));
   RopeTable rt = rope_layout(m.block.grid_f, m.block.grid_h, m.block.grid_w, m.block.d / std::max(1, m.block.heads));
@@ -156,8 +166,13 @@ acid_status validate_model(const acid_model& m) {
 
 acid_status validate_cfg(const acid_loop_cfg& c) {
   ACID_REQUIRE(c.n_steps > 0 && c.warmup >= 0, ACID_ERR_INVALID_ARG, "loop: n_steps must be > 0, warmup >= 0");
-  ACID_REQUIRE(c.method == ACID_METHOD_TEACACHE || c.method == ACID_METHOD_EASYCACHE, ACID_ERR_INVALID_ARG,
-               "loop: unknown method");
+  ACID_REQUIRE(c.method == ACID_METHOD_TEACACHE || c.method == ACID_METHOD_EASYCACHE ||
+                   c.method == ACID_METHOD_DICACHE,
+               ACID_ERR_INVALID_ARG, "loop: unknown method");
+  ACID_REQUIRE(c.method != ACID_METHOD_DICACHE || c.probe_blocks >= 1, ACID_ERR_INVALID_ARG,
+               "loop: DiCache needs probe_blocks >= 1");
+  ACID_REQUIRE(c.method == ACID_METHOD_EASYCACHE || c.warmup >= 1, ACID_ERR_INVALID_ARG,
+               "loop: TeaCache and DiCache need warmup >= 1 (the first signal compares two steps)");
   ACID_REQUIRE(c.method != ACID_METHOD_EASYCACHE || c.warmup >= 2, ACID_ERR_INVALID_ARG,
                "loop: EasyCache needs warmup >= 2 (k is defined after two computed steps)");
   ACID_REQUIRE(c.shift > 0.0, ACID_ERR_INVALID_ARG, "loop: shift must be > 0");
@@ -209,18 +224,90 @@ acid_status read_results(double* host, const double* dev, int n, cudaStream_t s)
 }
 
 // Runs every block on the state in w.xbuf.
-acid_status run_blocks(const acid_model& m, const LoopWs& w, cudaStream_t s) {
+acid_status run_blocks(const acid_model& m, const LoopWs& w, cudaStream_t s, int b0 = 0, int b1 = -1) {
   const RopeTable base_rope = [&] {
     RopeTable t = rope_layout(m.block.grid_f, m.block.grid_h, m.block.grid_w, m.block.d / m.block.heads);
     t.table = w.rope;
     return t;
   }();
   const void* ctx = m.block.kind == ACID_BLOCK_WAN && m.block.n_text > 0 ? w.text : nullptr;
-  for (int i = 0; i < total_blocks(m); ++i) {
+  if (b1 < 0) b1 = total_blocks(m);
+  for (int i = b0; i < b1; ++i) {
     const acid_block_desc d = desc_for(m, i);
     const BlockWs bws = block_ws_layout(d, w.block_base);
     ACID_TRY(block_forward_impl(d, w.xbuf, w.temb, ctx, m.blocks[i], bws, &base_rope, s));
   }
+  return ACID_OK;
+}
+
+// ---------------------------------------------------------------- DiCache
+// After a computed step: D = H_out - P_t; the caches shift
+// (P_2, D_2) <- (P_1, D_1), (P_1, D_1) <- (P_t, D); on the first computed
+// step both slots get (P_t, D), so the trajectory term vanishes.
+template <typename T>
+__global__ void dicache_update_kernel(const T* __restrict__ h_out, const float* __restrict__ p_t, float* d1,
+                                      float* d2, float* p1, float* p2, int64_t n, const int* count) {
+  const int c = *count;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float p = p_t[i];
+    const float d = io<T>::ld(h_out + i) - p;
+    if (c >= 1) {
+      d2[i] = d1[i];
+      p2[i] = p1[i];
+    } else {
+      d2[i] = d;
+      p2[i] = p;
+    }
+    d1[i] = d;
+    p1[i] = p;
+  }
+}
+
+__global__ void dicache_count_kernel(int* count) { *count = min(*count + 1, 2); }
+
+// Reuse: H_out = P_t + D_1 + g (D_1 - D_2), g = sum|P_t - P_1| / sum|P_1 - P_2|
+// (0 when the denominator is 0); the sums are read from device memory.
+template <typename T>
+__global__ void dicache_reuse_kernel(T* out, const float* __restrict__ p_t, const float* __restrict__ d1,
+                                     const float* __restrict__ d2, int64_t n, const double* num, const double* den) {
+  const double dn = *den;
+  const float g = dn > 0.0 ? (float)(*num / dn) : 0.0f;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float a = d1[i];
+    io<T>::st(out + i, p_t[i] + a + g * (a - d2[i]));
+  }
+}
+
+int elem_grid(int64_t n) { return (int)std::min<int64_t>(152 * 16, std::max<int64_t>(1, (n + 255) / 256)); }
+
+acid_status dicache_update(int dt, const void* h_out, const float* p_t, const LoopWs& w, int64_t n, cudaStream_t s) {
+  if (dt == ACID_BF16)
+    dicache_update_kernel<__nv_bfloat16><<<elem_grid(n), 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(h_out), p_t, w.resid, w.dc_d2, w.dc_p1, w.dc_p2, n, w.dc_count);
+  else
+    dicache_update_kernel<float><<<elem_grid(n), 256, 0, s>>>(static_cast<const float*>(h_out), p_t, w.resid,
+                                                              w.dc_d2, w.dc_p1, w.dc_p2, n, w.dc_count);
+  ACID_CHECK_LAUNCH();
+  dicache_count_kernel<<<1, 1, 0, s>>>(w.dc_count);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+// Reuse into out (the block-stack state's video rows, model dtype).  Uses
+// w.dres[0..5] for the two trajectory sums.
+acid_status dicache_reuse(int dt, void* out, const float* p_t, const LoopWs& w, int64_t n, cudaStream_t s) {
+  ACID_TRY(drift_launch(ACID_FP32, w.dc_p1, p_t, nullptr, nullptr, n, w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+  ACID_TRY(drift_launch(ACID_FP32, w.dc_p2, w.dc_p1, nullptr, nullptr, n, w.dres + 3, w.drift_ws,
+                        drift_workspace_bytes(0), s));
+  if (dt == ACID_BF16)
+    dicache_reuse_kernel<__nv_bfloat16><<<elem_grid(n), 256, 0, s>>>(static_cast<__nv_bfloat16*>(out), p_t, w.resid,
+                                                                     w.dc_d2, n, w.dres + 1, w.dres + 4);
+  else
+    dicache_reuse_kernel<float><<<elem_grid(n), 256, 0, s>>>(static_cast<float*>(out), p_t, w.resid, w.dc_d2, n,
+                                                            w.dres + 1, w.dres + 4);
+  ACID_CHECK_LAUNCH();
   return ACID_OK;
 }
 
@@ -287,6 +374,9 @@ extern "C" acid_status acid_loop_begin(const acid_model* m, const acid_loop_cfg*
   }
   RopeTable rt = rope_layout(m->block.grid_f, m->block.grid_h, m->block.grid_w, m->block.d / m->block.heads);
   ACID_TRY(rope_build(rt, w.rope, m->block.rope_theta, s));
+  ACID_CUDA(cudaMemsetAsync(w.dc_count, 0, sizeof(int), s));
+  ACID_REQUIRE(cfg->method != ACID_METHOD_DICACHE || cfg->probe_blocks <= total_blocks(*m), ACID_ERR_INVALID_ARG,
+               "acid_loop_begin: probe_blocks exceeds the number of blocks");
   return ACID_OK;
 }
 
@@ -369,6 +459,32 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
       st->have_cache = 1;
     } else {
       ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s));
+    }
+    ACID_TRY(final_layer(*m, w, x_video, nullptr, latent, dsig, s));
+  } else if (cfg->method == ACID_METHOD_DICACHE) {
+    // probe: the first probe_blocks blocks on every step; P_i (fp32) in temni[i & 1]
+    const int pb = cfg->probe_blocks;
+    float* p_cur = w.temni[i & 1];
+    float* p_prev = w.temni[(i & 1) ^ 1];
+    if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
+    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
+    ACID_TRY(run_blocks(*m, w, s, 0, pb));
+    ACID_TRY(add_mixed(dt, x_video, dt, x_video, ACID_FP32, p_cur, sh.N * sh.d, 0.0f, s));
+    if (!warm) {
+      ACID_REQUIRE(i > 0, ACID_ERR_INVALID_ARG, "DiCache needs at least one warmup step");
+      ACID_TRY(drift_launch(ACID_FP32, p_prev, p_cur, nullptr, nullptr, sh.N * sh.d, w.dres, w.drift_ws,
+                            drift_workspace_bytes(0), s));
+      double h[3];
+      ACID_TRY(read_results(h, w.dres, 3, s));
+      compute = controller_step(*st, *cfg, h[0], forced, &lg);
+    }
+    if (compute || !st->have_cache) {
+      compute = true;
+      ACID_TRY(run_blocks(*m, w, s, pb, total_blocks(*m)));
+      ACID_TRY(dicache_update(dt, x_video, p_cur, w, sh.N * sh.d, s));
+      st->have_cache = 1;
+    } else {
+      ACID_TRY(dicache_reuse(dt, x_video, p_cur, w, sh.N * sh.d, s));
     }
     ACID_TRY(final_layer(*m, w, x_video, nullptr, latent, dsig, s));
   } else {
@@ -466,7 +582,7 @@ __global__ void controller_kernel(DevLoop* st, const double* dres, const double*
   lg.ms = NAN;
   bool compute = true;
   if (!warm) {
-    const double s = st->method == ACID_METHOD_TEACACHE
+    const double s = st->method != ACID_METHOD_EASYCACHE
                          ? dres[0]
                          : dev_ratio_or_inf(st->k_rate * (dres[1] / st->latent_n), dres[5] / st->latent_n);
     st->sigma_acc += s;
@@ -565,10 +681,21 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
   // ---- signal and decision
   float* v = w.v[0];
   float* v_prev = w.v[1];
+  // DiCache probe features: current in temni[0], previous step's in temni[1]
+  float* p_cur = w.temni[0];
+  float* p_prev = w.temni[1];
+  const int pb = cfg.probe_blocks;
   if (cfg.method == ACID_METHOD_TEACACHE) {
     ACID_TRY(gemv(dt, m.blocks[0].mod.w, m.blocks[0].mod.b, w.temb, w.mod0, 2 * sh.d, sh.d, true, s));
     ACID_TRY(ln_mod_drift(w.h_in, w.temni[0], w.temni[1], step, 0, sh.N, sh.d, w.mod0, w.mod0 + sh.d, m.block.ln_eps,
                           w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+  } else if (cfg.method == ACID_METHOD_DICACHE) {
+    if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
+    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
+    ACID_TRY(run_blocks(m, w, s, 0, pb));
+    ACID_TRY(add_mixed(dt, x_video, dt, x_video, ACID_FP32, p_cur, sh.N * sh.d, 0.0f, s));
+    ACID_TRY(drift_launch(ACID_FP32, p_prev, p_cur, nullptr, nullptr, sh.N * sh.d, w.dres, w.drift_ws,
+                          drift_workspace_bytes(0), s));
   } else {
     ACID_TRY(drift_launch(ACID_FP32, w.x_prev, latent, nullptr, nullptr, sh.latent, w.dres, w.drift_ws,
                           drift_workspace_bytes(0), s));
@@ -582,10 +709,16 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
 
   // ---- compute body: the model
   ACID_CUDA(cudaStreamBeginCaptureToGraph(s2, br[0], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-  if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s2));
-  ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s2));
-  ACID_TRY(run_blocks(m, w, s2));
-  if (cfg.method == ACID_METHOD_TEACACHE) {
+  if (cfg.method == ACID_METHOD_DICACHE) {
+    ACID_TRY(run_blocks(m, w, s2, pb, total_blocks(m)));
+    ACID_TRY(dicache_update(dt, x_video, p_cur, w, sh.N * sh.d, s2));
+  } else {
+    if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s2));
+    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s2));
+    ACID_TRY(run_blocks(m, w, s2));
+  }
+  if (cfg.method == ACID_METHOD_DICACHE) {
+  } else if (cfg.method == ACID_METHOD_TEACACHE) {
     ACID_TRY(add_mixed(dt, x_video, ACID_FP32, w.h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s2));
   } else {
     ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s2));
@@ -603,6 +736,8 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
   ACID_CUDA(cudaStreamBeginCaptureToGraph(s2, br[1], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
   if (cfg.method == ACID_METHOD_TEACACHE)
     ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s2));
+  else if (cfg.method == ACID_METHOD_DICACHE)
+    ACID_TRY(dicache_reuse(dt, x_video, p_cur, w, sh.N * sh.d, s2));
   else
     ACID_TRY(add_mixed(ACID_FP32, latent, ACID_FP32, w.offset, ACID_FP32, v, sh.latent, 1.0f, s2));
   ACID_CUDA(cudaStreamEndCapture(s2, &tmp));
@@ -610,6 +745,9 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
   // ---- output: velocity and the Euler update, then the next step
   if (cfg.method == ACID_METHOD_TEACACHE) {
     ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s));
+  } else if (cfg.method == ACID_METHOD_DICACHE) {
+    ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s));
+    ACID_CUDA(cudaMemcpyAsync(p_prev, p_cur, sh.N * sh.d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   } else {
     ACID_CUDA(cudaMemcpyAsync(w.x_prev, latent, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
     ACID_CUDA(cudaMemcpyAsync(v_prev, v, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));

@@ -43,16 +43,18 @@ def _same_logs(la, lb):
             assert (np.isnan(x[k]) and np.isnan(y[k])) or x[k] == y[k], (k, x, y)
 
 
-@pytest.mark.parametrize("method", ["teacache", "easycache"])
+@pytest.mark.parametrize("method", ["teacache", "easycache", "dicache"])
 def test_toy_graph_equals_host_loop_and_oracle(acid, method):
     over = dict(method="easycache", tau_low=0.02, tau_high=0.04) if method == "easycache" else {}
+    if method == "dicache":
+        over = dict(method="dicache")
     cfg = S.get_config("toy", **over)
     w = S.model_weights(cfg, 5)
     lat = S.latent(cfg, 5)
     host, graph, la, lb = _both(acid, cfg, w, lat, method=method)
     _same_logs(la, lb)
     np.testing.assert_array_equal(graph, host)
-    ref = O.denoise_loop(cfg, w, lat, None)
+    ref = O.denoise_loop(cfg, w, lat, None, method=method)
     assert [bool(x["computed"]) for x in lb] == ref.computed
     assert np.abs(graph - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
     assert 0 < sum(ref.computed) < cfg.steps
@@ -69,8 +71,11 @@ def test_toy_graph_forced_and_force_last(acid):
     assert [x["computed"] for x in lb] == [1, 0, 1, 0, 0, 0, 1]
 
 
-@pytest.mark.parametrize("kind", ["wan", "cog", "hv"])
+@pytest.mark.parametrize("kind", ["wan", "cog", "hv", "hv-dicache"])
 def test_bf16_graph_equals_host_loop(acid, kind):
+    method = None
+    if kind == "hv-dicache":
+        kind, method = "hv", "dicache"
     over = dict(d=256, heads=2, ffn=512, latent_f=3, latent_h=16, latent_w=22, steps=8)
     if kind == "wan":
         cfg = S.get_config("wan", n_blocks=2, n_text=40, d_text=256, **over)
@@ -80,6 +85,7 @@ def test_bf16_graph_equals_host_loop(acid, kind):
     else:
         cfg = S.get_config("hv", n_blocks=1, n_single=1, n_text=30, d_text=256, **over)
     w = S.model_weights(cfg, 7)
-    host, graph, la, lb = _both(acid, cfg, w, S.latent(cfg, 7), S.text(cfg, 7))
+    kw = {} if method is None else dict(method=method, probe_blocks=1, tau_low=0.05, tau_high=0.2)
+    host, graph, la, lb = _both(acid, cfg, w, S.latent(cfg, 7), S.text(cfg, 7), **kw)
     _same_logs(la, lb)
     np.testing.assert_array_equal(graph, host)

@@ -52,7 +52,7 @@ def _compare_loop(acid, cfg, w, lat, text=None, **kw):
     logs = acid.acid_denoise_loop(model, c, tl, tt)
     acid.check_device_error()
     gpu_dec = [bool(l["computed"]) for l in logs]
-    okw = {k: v for k, v in kw.items() if k in ("tau_low", "tau_high", "delta", "method", "n_steps")}
+    okw = {k: v for k, v in kw.items() if k in ("tau_low", "tau_high", "delta", "method", "n_steps", "probe_blocks")}
     ref = O.denoise_loop(cfg, w, lat, text, **okw)
     forced = [None] * len(gpu_dec)
     for i in range(len(gpu_dec)):
@@ -93,6 +93,20 @@ def test_toy_loop_easycache(acid):
     lat = S.latent(cfg, 2)
     got, ref, _ = _compare_loop(acid, cfg, w, lat, method="easycache")
     assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+
+
+@pytest.mark.parametrize("probe_blocks,tau", [(1, (0.05, 0.2)), (1, (0.02, 0.04)), (2, (1e9, 1e9))])
+def test_toy_loop_dicache(acid, probe_blocks, tau):
+    """DiCache (probe-feature drift, trajectory reuse) against the oracle; a
+    probe as deep as the stack makes every reuse exact."""
+    cfg = S.get_config("toy", steps=10)
+    w = S.model_weights(cfg, 12)
+    lat = S.latent(cfg, 12)
+    got, ref, _ = _compare_loop(acid, cfg, w, lat, method="dicache", probe_blocks=probe_blocks, tau_low=tau[0],
+                                tau_high=tau[1])
+    assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+    if tau[0] < 1:
+        assert 0 < sum(ref.computed) < cfg.steps
 
 
 def test_toy_loop_forced_decisions(acid):
