@@ -294,6 +294,10 @@ typedef struct {
   double shift;              /* sigma shift s (1 = none) */
   const int8_t* forced;      /* host [n_steps] or NULL: -1 controller, 0 reuse, 1 compute */
   int32_t probe_blocks;      /* DiCache: blocks run on every step as the probe (>= 1) */
+  int32_t signal_poly_n;     /* 0: raw signal; else coefficients in signal_poly (<= 8) */
+  const double* signal_poly; /* host [signal_poly_n], ascending powers: the controller
+                                sees s' = sum_j c_j s^j (TeaCache's calibrated rescaling
+                                of its raw drift; not part of Algorithm 1 itself) */
 } acid_loop_cfg;
 
 typedef struct {

@@ -182,6 +182,16 @@ class AcidController:
         return skip, tau, sigma_seen, ds
 
 
+def rescale_signal(s: float, coeffs=None) -> float:
+    """Optional rescaling of a raw drift value before Algorithm 1,
+    s' = sum_j c_j s^j (ascending powers; identity without coefficients).
+    TeaCache calibrates such a polynomial per model; the paper's Algorithm 1
+    takes the base method's signal as given, so the default is the identity."""
+    if not coeffs:
+        return float(s)
+    return float(sum(c * s ** j for j, c in enumerate(coeffs)))
+
+
 def controller_decisions(signals, warmup: int, tau_low: float, tau_high: float,
                          delta: float) -> list[bool]:
     """Computed-step mask of Algorithm 1 for a fixed signal sequence
@@ -622,7 +632,7 @@ class LoopResult:
 
 def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None, delta=None,
                  warmup=None, method=None, forced=None, force_last=False, shift=1.0,
-                 probe_blocks=1) -> LoopResult:
+                 probe_blocks=1, signal_poly=None) -> LoopResult:
     """The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler
     flow-matching sampler, with TeaCache, EasyCache or DiCache as the base
     method M.
@@ -671,7 +681,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
             if i < warmup:
                 compute = True
             else:
-                s = rel_l1(temni_prev, temni)
+                s = rescale_signal(rel_l1(temni_prev, temni), signal_poly)
                 skip, tau, sg, ds = ctl.step(s, forced=f)
                 rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
                 compute = not skip
@@ -687,7 +697,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
             if i < warmup:
                 compute = True
             else:
-                s = easycache_signal(k_rate, x, x_prev, v_prev)
+                s = rescale_signal(easycache_signal(k_rate, x, x_prev, v_prev), signal_poly)
                 skip, tau, sg, ds = ctl.step(s, forced=f)
                 rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
                 compute = not skip
@@ -708,7 +718,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
             if i < warmup:
                 compute = True
             else:
-                s = rel_l1(probe_prev, probe)
+                s = rescale_signal(rel_l1(probe_prev, probe), signal_poly)
                 skip, tau, sg, ds = ctl.step(s, forced=f)
                 rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
                 compute = not skip

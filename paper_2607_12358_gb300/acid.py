@@ -296,7 +296,7 @@ _METHOD = {"teacache": A.ACID_METHOD_TEACACHE, "easycache": A.ACID_METHOD_EASYCA
 
 
 def loop_cfg(cfg, n_steps=None, tau_low=None, tau_high=None, delta=None, warmup=None, method=None,
-             force_last=False, shift=1.0, forced=None, probe_blocks=1):
+             force_last=False, shift=1.0, forced=None, probe_blocks=1, signal_poly=None):
     """acid_loop_cfg from a workload config; returns (struct, keepalive)."""
     method = cfg.method if method is None else method
     c = A.acid_loop_cfg()
@@ -309,10 +309,16 @@ def loop_cfg(cfg, n_steps=None, tau_low=None, tau_high=None, delta=None, warmup=
     c.tau_high = cfg.tau_high if tau_high is None else tau_high
     c.delta = cfg.delta if delta is None else delta
     c.shift = shift
-    keep = None
+    keep = []
     if forced is not None:
-        keep = (C.c_int8 * c.n_steps)(*[-1 if f is None else int(bool(f)) for f in forced])
-        c.forced = C.cast(keep, C.POINTER(C.c_int8))
+        fk = (C.c_int8 * c.n_steps)(*[-1 if f is None else int(bool(f)) for f in forced])
+        c.forced = C.cast(fk, C.POINTER(C.c_int8))
+        keep.append(fk)
+    if signal_poly is not None:
+        pk = (C.c_double * len(signal_poly))(*[float(x) for x in signal_poly])
+        c.signal_poly_n = len(signal_poly)
+        c.signal_poly = C.cast(pk, C.POINTER(C.c_double))
+        keep.append(pk)
     return c, keep
 
 

@@ -64,6 +64,8 @@ struct DevLoop {
   double sigma_acc, s_prev, k_rate;
   double tau_low, tau_high, delta;
   double latent_n;
+  int poly_n;
+  double poly[8];
 };
 
 struct Shape {
@@ -176,6 +178,8 @@ acid_status validate_cfg(const acid_loop_cfg& c) {
   ACID_REQUIRE(c.method != ACID_METHOD_EASYCACHE || c.warmup >= 2, ACID_ERR_INVALID_ARG,
                "loop: EasyCache needs warmup >= 2 (k is defined after two computed steps)");
   ACID_REQUIRE(c.shift > 0.0, ACID_ERR_INVALID_ARG, "loop: shift must be > 0");
+  ACID_REQUIRE(c.signal_poly_n >= 0 && c.signal_poly_n <= 8 && (c.signal_poly_n == 0 || c.signal_poly != nullptr),
+               ACID_ERR_INVALID_ARG, "loop: signal_poly_n must be 0..8 with coefficients given");
   return ACID_OK;
 }
 
@@ -187,7 +191,16 @@ double sigma_at(const acid_loop_cfg& c, int i) {
 
 // Algorithm 1, the non-warmup branch: accumulate, pick the threshold from the
 // signal's rate of change, compare, reset on compute; s_prev always updated.
-bool controller_step(acid_loop_state& st, const acid_loop_cfg& c, double s, int forced, acid_step_log* lg) {
+// Optional rescaling of the raw signal, s' = sum_j c_j s^j (Horner).
+__host__ __device__ inline double rescale_signal(double s, const double* c, int n) {
+  if (n <= 0) return s;
+  double r = c[n - 1];
+  for (int j = n - 2; j >= 0; --j) r = r * s + c[j];
+  return r;
+}
+
+bool controller_step(acid_loop_state& st, const acid_loop_cfg& c, double s_raw, int forced, acid_step_log* lg) {
+  const double s = rescale_signal(s_raw, c.signal_poly, c.signal_poly_n);
   st.sigma_acc += s;
   double tau, ds = NAN;
   if (st.have_prev_signal) {
@@ -582,9 +595,10 @@ __global__ void controller_kernel(DevLoop* st, const double* dres, const double*
   lg.ms = NAN;
   bool compute = true;
   if (!warm) {
-    const double s = st->method != ACID_METHOD_EASYCACHE
-                         ? dres[0]
-                         : dev_ratio_or_inf(st->k_rate * (dres[1] / st->latent_n), dres[5] / st->latent_n);
+    const double s_raw = st->method != ACID_METHOD_EASYCACHE
+                             ? dres[0]
+                             : dev_ratio_or_inf(st->k_rate * (dres[1] / st->latent_n), dres[5] / st->latent_n);
+    const double s = rescale_signal(s_raw, st->poly, st->poly_n);
     st->sigma_acc += s;
     double tau, ds = NAN;
     if (st->have_prev) {
@@ -787,6 +801,8 @@ extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_l
   d.tau_high = cfg->tau_high;
   d.delta = cfg->delta;
   d.latent_n = (double)sh.latent;
+  d.poly_n = cfg->signal_poly_n;
+  for (int j = 0; j < cfg->signal_poly_n; ++j) d.poly[j] = cfg->signal_poly[j];
   double sig[kMaxGraphSteps + 1];
   for (int i = 0; i <= cfg->n_steps; ++i) sig[i] = sigma_at(*cfg, i);
   ACID_CUDA(cudaMemcpyAsync(w.dev, &d, sizeof(d), cudaMemcpyHostToDevice, s));

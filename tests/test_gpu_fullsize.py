@@ -149,6 +149,36 @@ def test_wan_step_drift_decision_and_apply(acid):
         assert rel <= 2e-2, (i, rel)
 
 
+def test_hv_step_drift_and_decision(acid):
+    """HunyuanVideo shape (256 + 67320 tokens, d = 3072), one dual and one
+    single block: the TeaCache signal of step 1 teacher-forced from the GPU
+    latents, and the decision replayed through the oracle controller."""
+    cfg = S.get_config("hv", n_blocks=1, n_single=1, steps=50)
+    w = S.model_weights(cfg, 41)
+    lat = S.latent(cfg, 41)
+    text = S.text(cfg, 41)
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg, n_steps=cfg.steps)
+    loop = acid.Loop(model, c, torch.from_numpy(text).to(DEV, torch.bfloat16), DEV)
+    tl = torch.from_numpy(lat).to(DEV)
+    xs, logs = [tl.cpu().numpy().astype(np.float64)], []
+    for _ in range(2):
+        logs.append(acid.log_to_dict(loop.step(tl)))
+        xs.append(tl.cpu().numpy().astype(np.float64))
+    acid.check_device_error()
+    assert np.isfinite(xs[-1]).all()
+    sig = O.sigmas(cfg.steps)
+    temni = []
+    for i in range(2):
+        t = 1000 * sig[i]
+        si = O.step_inputs(cfg, w, xs[i], t, with_blocks=False)
+        temni.append(O.block0_temni(cfg, w, si.h_in, si.temb))
+    s_ref = O.rel_l1(temni[0], temni[1])
+    assert abs(logs[1]["signal"] - s_ref) <= 1e-3 * s_ref
+    skip, tau, sg, _ = O.AcidController(cfg.tau_low, cfg.tau_high, cfg.delta).step(logs[1]["signal"])
+    assert bool(logs[1]["computed"]) == (not skip) and logs[1]["tau"] == tau
+
+
 def test_cog_easycache_step_signal(acid):
     cfg = S.get_config("cog", n_blocks=1, steps=50)
     w = S.model_weights(cfg, 31)

@@ -60,6 +60,14 @@ def test_toy_graph_equals_host_loop_and_oracle(acid, method):
     assert 0 < sum(ref.computed) < cfg.steps
 
 
+def test_toy_graph_rescaled_signal(acid):
+    cfg = S.get_config("toy")
+    w = S.model_weights(cfg, 14)
+    host, graph, la, lb = _both(acid, cfg, w, S.latent(cfg, 14), signal_poly=[0.002, 1.5, 4.0])
+    _same_logs(la, lb)
+    np.testing.assert_array_equal(graph, host)
+
+
 def test_toy_graph_forced_and_force_last(acid):
     cfg = S.get_config("toy", steps=7)
     w = S.model_weights(cfg, 6)

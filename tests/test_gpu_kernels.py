@@ -76,6 +76,19 @@ def test_linear_bf16_epilogues(acid, epi):
     assert _rel_l2(got, ref) <= 4e-3
 
 
+@pytest.mark.parametrize("M,K,N", [(1, 64, 64), (7, 8, 32), (127, 72, 96), (129, 200, 256), (3, 4104, 128)])
+def test_linear_bf16_edge_shapes(acid, M, K, N):
+    """Single rows, K below / not a multiple of the 64-wide k-block (zero-filled
+    by TMA), N a multiple of 32 only, and a ragged long K."""
+    rng = np.random.default_rng(M * 1000 + K)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.1 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    got = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), out_fp32=True).cpu().numpy()
+    ref = O.linear(a, w, b)
+    assert np.abs(got - ref).max() <= 1e-4 * (1 + np.abs(ref).max())
+
+
 def test_linear_fp32(acid):
     M, K, N = 77, 96, 130
     rng = np.random.default_rng(8)

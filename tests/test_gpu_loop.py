@@ -52,7 +52,8 @@ def _compare_loop(acid, cfg, w, lat, text=None, **kw):
     logs = acid.acid_denoise_loop(model, c, tl, tt)
     acid.check_device_error()
     gpu_dec = [bool(l["computed"]) for l in logs]
-    okw = {k: v for k, v in kw.items() if k in ("tau_low", "tau_high", "delta", "method", "n_steps", "probe_blocks")}
+    okw = {k: v for k, v in kw.items()
+           if k in ("tau_low", "tau_high", "delta", "method", "n_steps", "probe_blocks", "signal_poly")}
     ref = O.denoise_loop(cfg, w, lat, text, **okw)
     forced = [None] * len(gpu_dec)
     for i in range(len(gpu_dec)):
@@ -107,6 +108,17 @@ def test_toy_loop_dicache(acid, probe_blocks, tau):
     assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
     if tau[0] < 1:
         assert 0 < sum(ref.computed) < cfg.steps
+
+
+@pytest.mark.parametrize("method", ["teacache", "easycache"])
+def test_toy_loop_rescaled_signal(acid, method):
+    """TeaCache-style polynomial rescaling of the raw signal before Algorithm 1."""
+    over = dict(method="easycache", tau_low=0.02, tau_high=0.04) if method == "easycache" else {}
+    cfg = S.get_config("toy", **over)
+    w = S.model_weights(cfg, 13)
+    lat = S.latent(cfg, 13)
+    got, ref, logs = _compare_loop(acid, cfg, w, lat, method=method, signal_poly=[0.002, 1.5, 4.0])
+    assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
 
 
 def test_toy_loop_forced_decisions(acid):

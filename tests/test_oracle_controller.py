@@ -256,3 +256,36 @@ def test_dicache_negative_threshold_is_uncached():
     r = O.denoise_loop(cfg, w, lat, None, method="dicache", tau_low=-1.0, tau_high=-1.0)
     assert all(r.computed)
     np.testing.assert_allclose(r.latent, _plain_sampler(cfg, w, lat, cfg.steps), atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Signal rescaling hook (TeaCache-style polynomial; identity by default)
+# ---------------------------------------------------------------------------
+
+def test_rescale_polynomial_closed_forms():
+    assert O.rescale_signal(0.3) == 0.3 and O.rescale_signal(0.3, []) == 0.3
+    assert O.rescale_signal(0.3, [0.0, 2.0]) == 0.6
+    assert O.rescale_signal(0.5, [1.0, 0.0, 4.0]) == pytest.approx(2.0)
+    assert O.rescale_signal(2.0, [0.5]) == 0.5
+
+
+@pytest.mark.parametrize("method", ["teacache", "dicache"])
+def test_scaled_signal_with_scaled_thresholds_is_unchanged(method):
+    """Doubling the signal, both thresholds and delta leaves every comparison
+    of Algorithm 1 unchanged (doubling is exact in floating point)."""
+    cfg = S.get_config("toy", steps=8)
+    w = S.model_weights(cfg, 10)
+    lat = S.latent(cfg, 10)
+    a = O.denoise_loop(cfg, w, lat, None, method=method, delta=0.005)
+    b = O.denoise_loop(cfg, w, lat, None, method=method, delta=0.01, tau_low=2 * cfg.tau_low,
+                       tau_high=2 * cfg.tau_high, signal_poly=[0.0, 2.0])
+    assert a.computed == b.computed and 0 < sum(a.computed) < cfg.steps
+    np.testing.assert_array_equal(a.latent, b.latent)
+
+
+def test_constant_polynomial_fixes_the_schedule():
+    cfg = S.get_config("toy", steps=6)
+    w = S.model_weights(cfg, 11)
+    lat = S.latent(cfg, 11)
+    assert all(O.denoise_loop(cfg, w, lat, None, signal_poly=[1.0]).computed)
+    assert O.denoise_loop(cfg, w, lat, None, signal_poly=[0.0]).computed == [True] + [False] * 5
