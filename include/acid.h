@@ -298,6 +298,10 @@ typedef struct {
   const double* signal_poly; /* host [signal_poly_n], ascending powers: the controller
                                 sees s' = sum_j c_j s^j (TeaCache's calibrated rescaling
                                 of its raw drift; not part of Algorithm 1 itself) */
+  const double* tau_schedule;/* host [n_steps] or NULL: a finite entry fixes the threshold
+                                of that step (overriding the delta rule; a low-then-high
+                                schedule is the fixed transition-point dual threshold of
+                                Sec. 3.2); NaN entries keep the delta rule */
 } acid_loop_cfg;
 
 typedef struct {

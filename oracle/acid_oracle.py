@@ -152,7 +152,9 @@ class AcidController:
     Warmup steps run the model and touch neither Sigma nor s_prev.
     ``forced`` overrides the decision of step 3 (used only to continue a
     comparison past an ambiguous step); the state then follows the forced
-    branch.
+    branch.  ``tau_fixed`` (a number, not NaN) replaces the threshold of step
+    2: the fixed-schedule dual threshold of Sec. 3.2, which switches from a
+    low to a high threshold at a chosen step regardless of the signal.
     """
 
     def __init__(self, tau_low: float, tau_high: float, delta: float):
@@ -162,7 +164,8 @@ class AcidController:
         self.sigma = 0.0
         self.s_prev: float | None = None
 
-    def step(self, s_t: float, forced: bool | None = None) -> tuple[bool, float, float, float]:
+    def step(self, s_t: float, forced: bool | None = None,
+             tau_fixed: float | None = None) -> tuple[bool, float, float, float]:
         """Returns (skip, tau, sigma_compared, |s_t - s_prev| or nan)."""
         s_t = float(s_t)
         self.sigma = self.sigma + s_t
@@ -172,6 +175,8 @@ class AcidController:
         else:
             ds = math.nan
             tau = self.tau_low
+        if tau_fixed is not None and not math.isnan(tau_fixed):
+            tau = float(tau_fixed)
         sigma_seen = self.sigma
         skip = sigma_seen <= tau
         if forced is not None:
@@ -193,7 +198,7 @@ def rescale_signal(s: float, coeffs=None) -> float:
 
 
 def controller_decisions(signals, warmup: int, tau_low: float, tau_high: float,
-                         delta: float) -> list[bool]:
+                         delta: float, tau_schedule=None) -> list[bool]:
     """Computed-step mask of Algorithm 1 for a fixed signal sequence
     (``signals[i]`` is ignored for the first ``warmup`` steps)."""
     ctl = AcidController(tau_low, tau_high, delta)
@@ -202,7 +207,7 @@ def controller_decisions(signals, warmup: int, tau_low: float, tau_high: float,
         if i < warmup:
             out.append(True)
             continue
-        skip, _, _, _ = ctl.step(s)
+        skip, _, _, _ = ctl.step(s, tau_fixed=None if tau_schedule is None else tau_schedule[i])
         out.append(not skip)
     return out
 
@@ -632,7 +637,7 @@ class LoopResult:
 
 def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None, delta=None,
                  warmup=None, method=None, forced=None, force_last=False, shift=1.0,
-                 probe_blocks=1, signal_poly=None) -> LoopResult:
+                 probe_blocks=1, signal_poly=None, tau_schedule=None) -> LoopResult:
     """The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler
     flow-matching sampler, with TeaCache, EasyCache or DiCache as the base
     method M.
@@ -651,6 +656,8 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
 
     ``forced``: optional per-step list of None/True/False; True or False
     replaces the controller's decision at that step (compute / skip).
+    ``tau_schedule``: optional per-step thresholds (None or NaN: the delta
+    rule), see AcidController.
     """
     n_steps = cfg.steps if n_steps is None else n_steps
     tau_low = cfg.tau_low if tau_low is None else tau_low
@@ -674,6 +681,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
         rec = StepRecord(step=i, warmup=i < warmup)
         si = step_inputs(cfg, w, x, t)
         f = None if forced is None else forced[i]
+        tf = None if tau_schedule is None else tau_schedule[i]
         if force_last and i == n_steps - 1 and f is None:
             f = True
         if method == "teacache":
@@ -682,7 +690,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
                 compute = True
             else:
                 s = rescale_signal(rel_l1(temni_prev, temni), signal_poly)
-                skip, tau, sg, ds = ctl.step(s, forced=f)
+                skip, tau, sg, ds = ctl.step(s, forced=f, tau_fixed=tf)
                 rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
                 compute = not skip
                 rec.forced = f is not None
@@ -698,7 +706,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
                 compute = True
             else:
                 s = rescale_signal(easycache_signal(k_rate, x, x_prev, v_prev), signal_poly)
-                skip, tau, sg, ds = ctl.step(s, forced=f)
+                skip, tau, sg, ds = ctl.step(s, forced=f, tau_fixed=tf)
                 rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
                 compute = not skip
                 rec.forced = f is not None
@@ -719,7 +727,7 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
                 compute = True
             else:
                 s = rescale_signal(rel_l1(probe_prev, probe), signal_poly)
-                skip, tau, sg, ds = ctl.step(s, forced=f)
+                skip, tau, sg, ds = ctl.step(s, forced=f, tau_fixed=tf)
                 rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
                 compute = not skip
                 rec.forced = f is not None

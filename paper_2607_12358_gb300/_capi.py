@@ -56,7 +56,7 @@ class acid_loop_cfg(C.Structure):
     _fields_ = [("n_steps", C.c_int32), ("warmup", C.c_int32), ("method", C.c_int32), ("force_last", C.c_int32),
                 ("tau_low", C.c_double), ("tau_high", C.c_double), ("delta", C.c_double), ("shift", C.c_double),
                 ("forced", C.POINTER(C.c_int8)), ("probe_blocks", C.c_int32), ("signal_poly_n", C.c_int32),
-                ("signal_poly", C.POINTER(C.c_double))]
+                ("signal_poly", C.POINTER(C.c_double)), ("tau_schedule", C.POINTER(C.c_double))]
 
 
 class acid_step_log(C.Structure):

@@ -10,6 +10,7 @@ leaves all allocation to the caller.
 from __future__ import annotations
 
 import ctypes as C
+import math
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -262,6 +263,7 @@ class DeviceModel:
 
     def __init__(self, cfg, weights: dict, device="cuda"):
         self.cfg = cfg
+        self.device = torch.device(device)
         wdtype = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
         self.wdtype = wdtype
         types = (["hv_dual"] * cfg.n_blocks + ["hv_single"] * cfg.n_single) if cfg.kind == "hv" \
@@ -296,7 +298,7 @@ _METHOD = {"teacache": A.ACID_METHOD_TEACACHE, "easycache": A.ACID_METHOD_EASYCA
 
 
 def loop_cfg(cfg, n_steps=None, tau_low=None, tau_high=None, delta=None, warmup=None, method=None,
-             force_last=False, shift=1.0, forced=None, probe_blocks=1, signal_poly=None):
+             force_last=False, shift=1.0, forced=None, probe_blocks=1, signal_poly=None, tau_schedule=None):
     """acid_loop_cfg from a workload config; returns (struct, keepalive)."""
     method = cfg.method if method is None else method
     c = A.acid_loop_cfg()
@@ -319,6 +321,12 @@ def loop_cfg(cfg, n_steps=None, tau_low=None, tau_high=None, delta=None, warmup=
         c.signal_poly_n = len(signal_poly)
         c.signal_poly = C.cast(pk, C.POINTER(C.c_double))
         keep.append(pk)
+    if tau_schedule is not None:
+        if len(tau_schedule) != c.n_steps:
+            raise ValueError("tau_schedule needs one entry per step")
+        tk = (C.c_double * c.n_steps)(*[math.nan if x is None else float(x) for x in tau_schedule])
+        c.tau_schedule = C.cast(tk, C.POINTER(C.c_double))
+        keep.append(tk)
     return c, keep
 
 

@@ -49,6 +49,7 @@ struct LoopWs {
   struct DevLoop* dev;      // controller state and configuration
   double* sig;              // [kMaxGraphSteps + 1] noise levels
   int8_t* forced;           // [kMaxGraphSteps]
+  double* tau_sched;        // [kMaxGraphSteps] fixed thresholds (NaN: delta rule)
   acid_step_log* dlog;      // [kMaxGraphSteps]
   size_t bytes;
 };
@@ -59,7 +60,7 @@ constexpr int kMaxGraphSteps = 1024;
 struct DevLoop {
   int step;  // first member: the kernels read the step index through &dev->step
   int have_prev, have_cache, have_rate;
-  int n_steps, warmup, method, force_last, use_forced;
+  int n_steps, warmup, method, force_last, use_forced, use_tau_sched;
   int compute;
   double sigma_acc, s_prev, k_rate;
   double tau_low, tau_high, delta;
@@ -135,6 +136,7 @@ LoopWs loop_layout(const acid_model& m, void* base) {
   w.dev = b.take<DevLoop>(1);
   w.sig = b.take<double>(kMaxGraphSteps + 1);
   w.forced = b.take<int8_t>(kMaxGraphSteps);
+  w.tau_sched = b.take<double>(kMaxGraphSteps);
   w.dlog = b.take<acid_step_log>(kMaxGraphSteps);
   w.bytes = b.off + 1024;
   return w;
@@ -189,8 +191,6 @@ double sigma_at(const acid_loop_cfg& c, int i) {
   return c.shift * s / (1.0 + (c.shift - 1.0) * s);
 }
 
-// Algorithm 1, the non-warmup branch: accumulate, pick the threshold from the
-// signal's rate of change, compare, reset on compute; s_prev always updated.
 // Optional rescaling of the raw signal, s' = sum_j c_j s^j (Horner).
 __host__ __device__ inline double rescale_signal(double s, const double* c, int n) {
   if (n <= 0) return s;
@@ -199,30 +199,48 @@ __host__ __device__ inline double rescale_signal(double s, const double* c, int 
   return r;
 }
 
-bool controller_step(acid_loop_state& st, const acid_loop_cfg& c, double s_raw, int forced, acid_step_log* lg) {
-  const double s = rescale_signal(s_raw, c.signal_poly, c.signal_poly_n);
-  st.sigma_acc += s;
+// One non-warmup step of Algorithm 1 on (Sigma, s_prev), shared by the host
+// and device controllers: accumulate, pick the threshold from the signal's
+// rate of change, compare, reset Sigma on compute; s_prev always updated.  tau_fix: a finite value replaces the threshold the
+// delta rule would pick (a fixed threshold schedule, Sec. 3.2's transition
+// experiment); NaN keeps the rule.  forced >= 0 replaces the decision.
+// Returns true when the step computes.
+__host__ __device__ inline bool algorithm1_step(double& sigma_acc, double& s_prev, int& have_prev, double s,
+                                                double tau_low, double tau_high, double delta, double tau_fix,
+                                                int forced, acid_step_log* lg) {
+  sigma_acc += s;
   double tau, ds = NAN;
-  if (st.have_prev_signal) {
-    ds = fabs(s - st.s_prev);
-    tau = ds <= c.delta ? c.tau_high : c.tau_low;
+  if (have_prev) {
+    ds = fabs(s - s_prev);
+    tau = ds <= delta ? tau_high : tau_low;
   } else {
-    tau = c.tau_low;
+    tau = tau_low;
   }
-  const double seen = st.sigma_acc;
+  if (tau_fix == tau_fix) tau = tau_fix;
+  const double seen = sigma_acc;
   bool skip = seen <= tau;
   if (forced >= 0) skip = forced == 0;
-  if (!skip) st.sigma_acc = 0.0;
-  st.s_prev = s;
-  st.have_prev_signal = 1;
-  if (lg) {
-    lg->signal = s;
-    lg->dsignal = ds;
-    lg->tau = tau;
-    lg->sigma = seen;
-    lg->forced = forced >= 0;
-  }
+  if (!skip) sigma_acc = 0.0;
+  s_prev = s;
+  have_prev = 1;
+  lg->signal = s;
+  lg->dsignal = ds;
+  lg->tau = tau;
+  lg->sigma = seen;
+  lg->forced = forced >= 0;
   return !skip;
+}
+
+bool controller_step(acid_loop_state& st, const acid_loop_cfg& c, int i, double s_raw, int forced,
+                     acid_step_log* lg) {
+  const double s = rescale_signal(s_raw, c.signal_poly, c.signal_poly_n);
+  const double tau_fix = c.tau_schedule ? c.tau_schedule[i] : NAN;
+  int have_prev = st.have_prev_signal;
+  acid_step_log tmp;
+  const bool compute = algorithm1_step(st.sigma_acc, st.s_prev, have_prev, s, c.tau_low, c.tau_high, c.delta,
+                                       tau_fix, forced, lg ? lg : &tmp);
+  st.have_prev_signal = have_prev;
+  return compute;
 }
 
 double ratio_or_inf(double num, double den) {
@@ -463,7 +481,7 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
       ACID_REQUIRE(i > 0, ACID_ERR_INVALID_ARG, "TeaCache needs at least one warmup step");
       double h[3];
       ACID_TRY(read_results(h, w.dres, 3, s));
-      compute = controller_step(*st, *cfg, h[0], forced, &lg);
+      compute = controller_step(*st, *cfg, i, h[0], forced, &lg);
     }
     if (compute || !st->have_cache) {
       compute = true;
@@ -489,7 +507,7 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
                             drift_workspace_bytes(0), s));
       double h[3];
       ACID_TRY(read_results(h, w.dres, 3, s));
-      compute = controller_step(*st, *cfg, h[0], forced, &lg);
+      compute = controller_step(*st, *cfg, i, h[0], forced, &lg);
     }
     if (compute || !st->have_cache) {
       compute = true;
@@ -513,7 +531,7 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
       double h[6];
       ACID_TRY(read_results(h, w.dres, 6, s));
       const double sig_t = ratio_or_inf(st->k_rate * (h[1] / sh.latent), h[5] / sh.latent);
-      compute = controller_step(*st, *cfg, sig_t, forced, &lg);
+      compute = controller_step(*st, *cfg, i, sig_t, forced, &lg);
     }
     if (compute || !st->have_cache) {
       compute = true;
@@ -577,11 +595,12 @@ __device__ double dev_ratio_or_inf(double num, double den) {
   return num / den;
 }
 
-// Algorithm 1 on the device (one thread): same arithmetic as controller_step.
+// Algorithm 1 on the device (one thread), through the same algorithm1_step.
 // dres: TeaCache {rel, num, den}; EasyCache {., sum|x - x_prev|, .,
 // ., ., sum|v_prev|}.
 __global__ void controller_kernel(DevLoop* st, const double* dres, const double* sig, const int8_t* forced,
-                                  acid_step_log* log, cudaGraphConditionalHandle h_compute) {
+                                  const double* tau_sched, acid_step_log* log,
+                                  cudaGraphConditionalHandle h_compute) {
   const int i = st->step;
   const bool warm = i < st->warmup;
   int f = st->use_forced ? forced[i] : -1;
@@ -599,26 +618,9 @@ __global__ void controller_kernel(DevLoop* st, const double* dres, const double*
                              ? dres[0]
                              : dev_ratio_or_inf(st->k_rate * (dres[1] / st->latent_n), dres[5] / st->latent_n);
     const double s = rescale_signal(s_raw, st->poly, st->poly_n);
-    st->sigma_acc += s;
-    double tau, ds = NAN;
-    if (st->have_prev) {
-      ds = fabs(s - st->s_prev);
-      tau = ds <= st->delta ? st->tau_high : st->tau_low;
-    } else {
-      tau = st->tau_low;
-    }
-    const double seen = st->sigma_acc;
-    bool skip = seen <= tau;
-    if (f >= 0) skip = f == 0;
-    if (!skip) st->sigma_acc = 0.0;
-    st->s_prev = s;
-    st->have_prev = 1;
-    compute = !skip;
-    lg.signal = s;
-    lg.dsignal = ds;
-    lg.tau = tau;
-    lg.sigma = seen;
-    lg.forced = f >= 0;
+    const double tau_fix = st->use_tau_sched ? tau_sched[i] : NAN;
+    compute = algorithm1_step(st->sigma_acc, st->s_prev, st->have_prev, s, st->tau_low, st->tau_high, st->delta,
+                              tau_fix, f, &lg);
   }
   if (!st->have_cache) compute = true;
   if (compute) st->have_cache = 1;
@@ -716,7 +718,7 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
     ACID_TRY(drift_launch(ACID_FP32, v_prev, v_prev, nullptr, nullptr, sh.latent, w.dres + 3, w.drift_ws,
                           drift_workspace_bytes(0), s));
   }
-  controller_kernel<<<1, 1, 0, s>>>(w.dev, w.dres, w.sig, w.forced, w.dlog, h_compute);
+  controller_kernel<<<1, 1, 0, s>>>(w.dev, w.dres, w.sig, w.forced, w.tau_sched, w.dlog, h_compute);
   ACID_CHECK_LAUNCH();
   cudaGraph_t br[2];
   ACID_TRY(add_conditional(s, h_compute, cudaGraphCondTypeIf, 2, br));
@@ -797,6 +799,7 @@ extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_l
   d.method = cfg->method;
   d.force_last = cfg->force_last;
   d.use_forced = cfg->forced != nullptr;
+  d.use_tau_sched = cfg->tau_schedule != nullptr;
   d.tau_low = cfg->tau_low;
   d.tau_high = cfg->tau_high;
   d.delta = cfg->delta;
@@ -809,6 +812,9 @@ extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_l
   ACID_CUDA(cudaMemcpyAsync(w.sig, sig, sizeof(double) * (cfg->n_steps + 1), cudaMemcpyHostToDevice, s));
   if (cfg->forced)
     ACID_CUDA(cudaMemcpyAsync(w.forced, cfg->forced, cfg->n_steps, cudaMemcpyHostToDevice, s));
+  if (cfg->tau_schedule)
+    ACID_CUDA(cudaMemcpyAsync(w.tau_sched, cfg->tau_schedule, sizeof(double) * cfg->n_steps,
+                              cudaMemcpyHostToDevice, s));
   ACID_CUDA(cudaStreamSynchronize(s));  // host sources above are stack memory
 
   GraphCapture gc;

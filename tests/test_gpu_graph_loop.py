@@ -68,6 +68,15 @@ def test_toy_graph_rescaled_signal(acid):
     np.testing.assert_array_equal(graph, host)
 
 
+def test_toy_graph_transition_schedule(acid):
+    cfg = S.get_config("toy")
+    w = S.model_weights(cfg, 16)
+    sched = [cfg.tau_low] * 5 + [float("nan")] * 2 + [cfg.tau_high] * 3
+    host, graph, la, lb = _both(acid, cfg, w, S.latent(cfg, 16), tau_schedule=sched)
+    _same_logs(la, lb)
+    np.testing.assert_array_equal(graph, host)
+
+
 def test_toy_graph_forced_and_force_last(acid):
     cfg = S.get_config("toy", steps=7)
     w = S.model_weights(cfg, 6)

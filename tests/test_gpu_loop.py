@@ -53,7 +53,8 @@ def _compare_loop(acid, cfg, w, lat, text=None, **kw):
     acid.check_device_error()
     gpu_dec = [bool(l["computed"]) for l in logs]
     okw = {k: v for k, v in kw.items()
-           if k in ("tau_low", "tau_high", "delta", "method", "n_steps", "probe_blocks", "signal_poly")}
+           if k in ("tau_low", "tau_high", "delta", "method", "n_steps", "probe_blocks", "signal_poly",
+                     "tau_schedule")}
     ref = O.denoise_loop(cfg, w, lat, text, **okw)
     forced = [None] * len(gpu_dec)
     for i in range(len(gpu_dec)):
@@ -119,6 +120,18 @@ def test_toy_loop_rescaled_signal(acid, method):
     lat = S.latent(cfg, 13)
     got, ref, logs = _compare_loop(acid, cfg, w, lat, method=method, signal_poly=[0.002, 1.5, 4.0])
     assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+
+
+@pytest.mark.parametrize("k", [1, 4, 8])
+def test_toy_loop_transition_schedule(acid, k):
+    """Fixed low-to-high threshold schedule switching at step k (Sec. 3.2)."""
+    cfg = S.get_config("toy")
+    w = S.model_weights(cfg, 15)
+    lat = S.latent(cfg, 15)
+    sched = [cfg.tau_low] * k + [cfg.tau_high] * (cfg.steps - k)
+    got, ref, logs = _compare_loop(acid, cfg, w, lat, tau_schedule=sched)
+    assert np.abs(got - ref.latent).max() <= 1e-4 * np.abs(ref.latent).max()
+    assert [l["tau"] for l in logs[cfg.warmup:]] == sched[cfg.warmup:]
 
 
 def test_toy_loop_forced_decisions(acid):

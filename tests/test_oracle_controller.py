@@ -289,3 +289,58 @@ def test_constant_polynomial_fixes_the_schedule():
     lat = S.latent(cfg, 11)
     assert all(O.denoise_loop(cfg, w, lat, None, signal_poly=[1.0]).computed)
     assert O.denoise_loop(cfg, w, lat, None, signal_poly=[0.0]).computed == [True] + [False] * 5
+
+
+# ---------------------------------------------------------------------------
+# Fixed threshold schedule (the transition-point experiment of Sec. 3.2)
+# ---------------------------------------------------------------------------
+
+def test_schedule_worked_example():
+    """Worked by hand.  Signals 0.25 after one warmup step, delta = -1 (the
+    rule alone would always pick tau_low), schedule 0.4 before step 4 and 0.8
+    from step 4 on.  Sigma: 0.25 skip; 0.5 > 0.4 compute; 0.25 skip;
+    0.5 <= 0.8 skip; 0.75 skip; 1.0 > 0.8 compute."""
+    s = [0.0] + [0.25] * 6
+    sched = [0.4] * 4 + [0.8] * 3
+    d = O.controller_decisions(s, 1, 0.4, 0.8, -1.0, tau_schedule=sched)
+    assert d == [True, False, True, False, False, False, True]
+    ctl = O.AcidController(0.4, 0.8, -1.0)
+    taus = [ctl.step(x, tau_fixed=t)[1] for x, t in zip(s[1:], sched[1:])]
+    assert taus == sched[1:]
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_nan_schedule_is_algorithm1_and_constant_schedule_is_fixed_tau(seed):
+    rng = np.random.default_rng(300 + seed)
+    s = _random_signals(rng, 50)
+    tl, th = sorted(rng.uniform(0.02, 0.4, size=2))
+    delta = rng.uniform(0.0, 0.05)
+    assert O.controller_decisions(s, 1, tl, th, delta, tau_schedule=[math.nan] * 50) == \
+        O.controller_decisions(s, 1, tl, th, delta)
+    tau = rng.uniform(0.02, 0.4)
+    assert O.controller_decisions(s, 1, tl, th, delta, tau_schedule=[tau] * 50) == _fixed_tau(s, 1, tau)
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_transition_schedule_prefix_and_count(seed):
+    """Low until step k, high after: the controller is causal, so steps before
+    k decide as fixed tau_low does; the thresholds lie pointwise between the
+    two fixed ones, so the compute count does too (same greedy argument as
+    test_compute_count_between_fixed_thresholds)."""
+    rng = np.random.default_rng(400 + seed)
+    n = 50
+    s = _random_signals(rng, n)
+    tl, th = sorted(rng.uniform(0.02, 0.4, size=2))
+    k = int(rng.integers(1, n))
+    d = O.controller_decisions(s, 1, tl, th, 0.01, tau_schedule=[tl] * k + [th] * (n - k))
+    lo = _fixed_tau(s, 1, tl)
+    assert d[:k] == lo[:k]
+    assert sum(_fixed_tau(s, 1, th)) <= sum(d) <= sum(lo)
+
+
+def test_loop_schedule_of_low_threshold_is_fixed_low(toy):
+    cfg, w, lat = toy
+    a = O.denoise_loop(cfg, w, lat, None, tau_schedule=[cfg.tau_low] * cfg.steps)
+    b = O.denoise_loop(cfg, w, lat, None, tau_high=cfg.tau_low)
+    assert a.computed == b.computed
+    np.testing.assert_array_equal(a.latent, b.latent)
