@@ -11,7 +11,8 @@ Sections follow the paper:
 * the reverse-diffusion step loop (Sec. 3.1, Eq. 2), taken as Euler
   flow-matching steps because the workloads specify that sampler;
 * the DiT denoiser f_theta(x_t, t, c) (named, not defined, by the paper;
-  the block definitions below are readings, listed in the design doc).
+  the paper gives no block definition, so the ones below are readings of
+  the workloads' stated architecture).
 
 Parity pins live in ``tests/test_oracle_*.py``.
 """
@@ -635,12 +636,11 @@ class LoopResult:
         return [r.computed for r in self.records]
 
 
-def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None, delta=None,
-                 warmup=None, method=None, forced=None, force_last=False, shift=1.0,
-                 probe_blocks=1, signal_poly=None, tau_schedule=None) -> LoopResult:
-    """The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler
-    flow-matching sampler, with TeaCache, EasyCache or DiCache as the base
-    method M.
+class SamplerBranch:
+    """One stream of model evaluations inside the sampler, with its own
+    Algorithm 1 controller and its own cache of the base method M.  A plain
+    generation has one branch; classifier-free guidance has two (conditional
+    and unconditional text), which decide and cache independently.
 
     TeaCache (Sec. 2): s_t = rel_l1(TEMNI_{t-1}, TEMNI_t) between consecutive
     steps (computed or not); M.update stores R = H_out - H_in of the block
@@ -648,106 +648,168 @@ def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None
     EasyCache (Sec. 2): s_t = k * mean|x_t - x_{t-1}| / mean|v_{t-1}|;
     M.update refreshes k and the offset v_c - x_c; M.reuse gives
     v_t = x_t + (v_c - x_c).
-
     DiCache (Sec. 2): the first ``probe_blocks`` blocks run on every step;
     s_t = rel_l1(P_{t-1}, P_t) of the probe features; M.update keeps the probe
     features and deep parts D = H_out - P of the last two computed steps;
     M.reuse is dicache_reuse.
+    """
+
+    def __init__(self, cfg, w, text, tau_low, tau_high, delta, warmup, method, probe_blocks=1,
+                 signal_poly=None):
+        self.cfg, self.w = cfg, w
+        self.ctx = text_context(cfg, w, text)
+        self.ctl = AcidController(tau_low, tau_high, delta)
+        self.warmup, self.method = warmup, method
+        self.probe_blocks, self.signal_poly = probe_blocks, signal_poly
+        self.temni_prev = self.resid = None
+        self.x_prev = self.v_prev = self.x_c = self.v_c = self.k_rate = None
+        self.probe_prev = self.p_c1 = self.p_c2 = self.d_c1 = self.d_c2 = None
+
+    def _decide(self, rec, s, f, tf):
+        skip, tau, sg, ds = self.ctl.step(s, forced=f, tau_fixed=tf)
+        rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
+        rec.forced = f is not None
+        return not skip
+
+    def velocity(self, i, x, si, f=None, tf=None):
+        """The model output v at step i for latent x (si = step_inputs of x):
+        Algorithm 1 decides compute or reuse; returns (v, StepRecord).
+        f: forced decision (None, True, False); tf: fixed threshold or None."""
+        cfg, w, ctx, poly = self.cfg, self.w, self.ctx, self.signal_poly
+        rec = StepRecord(step=i, warmup=i < self.warmup)
+        if self.method == "teacache":
+            temni = block0_temni(cfg, w, si.h_in, si.temb)
+            compute = True if rec.warmup else \
+                self._decide(rec, rescale_signal(rel_l1(self.temni_prev, temni), poly), f, tf)
+            self.temni_prev = temni
+            if compute:
+                h_out = block_stack(cfg, w, si.h_in, si.mods, ctx)
+                self.resid = h_out - si.h_in
+            else:
+                h_out = cache_apply(si.h_in, self.resid)
+            v = final_layer(cfg, w, h_out, si.final_mod)
+        elif self.method == "easycache":
+            compute = True if rec.warmup else \
+                self._decide(rec, rescale_signal(easycache_signal(self.k_rate, x, self.x_prev, self.v_prev), poly),
+                             f, tf)
+            if compute:
+                h_out = block_stack(cfg, w, si.h_in, si.mods, ctx)
+                v = final_layer(cfg, w, h_out, si.final_mod)
+                if self.x_prev is not None:
+                    self.k_rate = easycache_rate(x, self.x_prev, v, self.v_prev)
+                self.x_c, self.v_c = x, v
+            else:
+                v = easycache_reuse(x, self.x_c, self.v_c)
+            self.x_prev, self.v_prev = x, v
+        elif self.method == "dicache":
+            # probe: the first probe_blocks blocks, run on every step
+            pb = self.probe_blocks
+            state = run_block_range(cfg, w, stack_state(cfg, si.h_in, ctx), si.mods, ctx, 0, pb)
+            probe = state_video(cfg, state, ctx)
+            compute = True if rec.warmup else \
+                self._decide(rec, rescale_signal(rel_l1(self.probe_prev, probe), poly), f, tf)
+            self.probe_prev = probe
+            if compute:
+                state = run_block_range(cfg, w, state, si.mods, ctx, pb, len(w["blocks"]))
+                h_out = state_video(cfg, state, ctx)
+                d_new = h_out - probe
+                if self.p_c1 is None:
+                    self.p_c2, self.d_c2 = probe, d_new
+                else:
+                    self.p_c2, self.d_c2 = self.p_c1, self.d_c1
+                self.p_c1, self.d_c1 = probe, d_new
+            else:
+                h_out = dicache_reuse(probe, self.p_c1, self.p_c2, self.d_c1, self.d_c2)
+            v = final_layer(cfg, w, h_out, si.final_mod)
+        else:
+            raise ValueError(self.method)
+        rec.computed = compute
+        return v, rec
+
+
+def _loop_args(cfg, n_steps, tau_low, tau_high, delta, warmup, method):
+    return (cfg.steps if n_steps is None else n_steps,
+            cfg.tau_low if tau_low is None else tau_low,
+            cfg.tau_high if tau_high is None else tau_high,
+            cfg.delta if delta is None else delta,
+            cfg.warmup if warmup is None else warmup,
+            cfg.method if method is None else method)
+
+
+def _step_override(seq, i):
+    return None if seq is None else seq[i]
+
+
+def denoise_loop(cfg, w, latent, text, n_steps=None, tau_low=None, tau_high=None, delta=None,
+                 warmup=None, method=None, forced=None, force_last=False, shift=1.0,
+                 probe_blocks=1, signal_poly=None, tau_schedule=None) -> LoopResult:
+    """The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler
+    flow-matching sampler, with TeaCache, EasyCache or DiCache as the base
+    method M (one SamplerBranch).
 
     ``forced``: optional per-step list of None/True/False; True or False
     replaces the controller's decision at that step (compute / skip).
     ``tau_schedule``: optional per-step thresholds (None or NaN: the delta
     rule), see AcidController.
     """
-    n_steps = cfg.steps if n_steps is None else n_steps
-    tau_low = cfg.tau_low if tau_low is None else tau_low
-    tau_high = cfg.tau_high if tau_high is None else tau_high
-    delta = cfg.delta if delta is None else delta
-    warmup = cfg.warmup if warmup is None else warmup
-    method = cfg.method if method is None else method
+    n_steps, tau_low, tau_high, delta, warmup, method = _loop_args(cfg, n_steps, tau_low, tau_high, delta, warmup,
+                                                                   method)
     sig = sigmas(n_steps, shift)
-    ctl = AcidController(tau_low, tau_high, delta)
-    ctx = text_context(cfg, w, text)
+    br = SamplerBranch(cfg, w, text, tau_low, tau_high, delta, warmup, method, probe_blocks, signal_poly)
     x = np.asarray(latent, F64)
     res = LoopResult(latent=x)
-    temni_prev = None
-    resid = None
-    x_prev = v_prev = None
-    x_c = v_c = None
-    k_rate = None
-    probe_prev = p_c1 = p_c2 = d_c1 = d_c2 = None
     for i in range(n_steps):
-        t = 1000.0 * sig[i]
-        rec = StepRecord(step=i, warmup=i < warmup)
-        si = step_inputs(cfg, w, x, t)
-        f = None if forced is None else forced[i]
-        tf = None if tau_schedule is None else tau_schedule[i]
+        si = step_inputs(cfg, w, x, 1000.0 * sig[i])
+        f = _step_override(forced, i)
         if force_last and i == n_steps - 1 and f is None:
             f = True
-        if method == "teacache":
-            temni = block0_temni(cfg, w, si.h_in, si.temb)
-            if i < warmup:
-                compute = True
-            else:
-                s = rescale_signal(rel_l1(temni_prev, temni), signal_poly)
-                skip, tau, sg, ds = ctl.step(s, forced=f, tau_fixed=tf)
-                rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
-                compute = not skip
-                rec.forced = f is not None
-            temni_prev = temni
-            if compute:
-                h_out = block_stack(cfg, w, si.h_in, si.mods, ctx)
-                resid = h_out - si.h_in
-            else:
-                h_out = cache_apply(si.h_in, resid)
-            v = final_layer(cfg, w, h_out, si.final_mod)
-        elif method == "easycache":
-            if i < warmup:
-                compute = True
-            else:
-                s = rescale_signal(easycache_signal(k_rate, x, x_prev, v_prev), signal_poly)
-                skip, tau, sg, ds = ctl.step(s, forced=f, tau_fixed=tf)
-                rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
-                compute = not skip
-                rec.forced = f is not None
-            if compute:
-                h_out = block_stack(cfg, w, si.h_in, si.mods, ctx)
-                v = final_layer(cfg, w, h_out, si.final_mod)
-                if x_prev is not None:
-                    k_rate = easycache_rate(x, x_prev, v, v_prev)
-                x_c, v_c = x, v
-            else:
-                v = easycache_reuse(x, x_c, v_c)
-            x_prev, v_prev = x, v
-        elif method == "dicache":
-            # probe: the first probe_blocks blocks, run on every step
-            state = run_block_range(cfg, w, stack_state(cfg, si.h_in, ctx), si.mods, ctx, 0, probe_blocks)
-            probe = state_video(cfg, state, ctx)
-            if i < warmup:
-                compute = True
-            else:
-                s = rescale_signal(rel_l1(probe_prev, probe), signal_poly)
-                skip, tau, sg, ds = ctl.step(s, forced=f, tau_fixed=tf)
-                rec.signal, rec.tau, rec.sigma, rec.dsignal = s, tau, sg, ds
-                compute = not skip
-                rec.forced = f is not None
-            probe_prev = probe
-            if compute:
-                state = run_block_range(cfg, w, state, si.mods, ctx, probe_blocks, len(w["blocks"]))
-                h_out = state_video(cfg, state, ctx)
-                d_new = h_out - probe
-                if p_c1 is None:
-                    p_c2, d_c2 = probe, d_new
-                else:
-                    p_c2, d_c2 = p_c1, d_c1
-                p_c1, d_c1 = probe, d_new
-            else:
-                h_out = dicache_reuse(probe, p_c1, p_c2, d_c1, d_c2)
-            v = final_layer(cfg, w, h_out, si.final_mod)
-        else:
-            raise ValueError(method)
-        rec.computed = compute
+        v, rec = br.velocity(i, x, si, f, _step_override(tau_schedule, i))
         res.records.append(rec)
         x = euler_step(x, v, sig[i], sig[i + 1])
     res.latent = x
     return res
+
+
+@dataclass
+class GuidedResult:
+    latent: np.ndarray
+    cond: list = field(default_factory=list)     # StepRecord per step, conditional branch
+    uncond: list = field(default_factory=list)   # StepRecord per step, unconditional branch
+
+
+def guided_velocity(v_cond, v_uncond, scale: float):
+    """Classifier-free guidance: v = v_u + g (v_c - v_u)."""
+    return v_uncond + scale * (v_cond - v_uncond)
+
+
+def denoise_loop_guided(cfg, w, latent, text_cond, text_uncond, scale, n_steps=None, tau_low=None, tau_high=None,
+                        delta=None, warmup=None, method=None, forced_cond=None, forced_uncond=None,
+                        force_last=False, shift=1.0, probe_blocks=1, signal_poly=None,
+                        tau_schedule=None) -> GuidedResult:
+    """Algorithm 1 with classifier-free guidance: the conditional and the
+    unconditional model evaluations are two SamplerBranches, each with its
+    own Sigma, s_prev and cache (the paper is silent on guidance; caching
+    the branches independently is the reading).  Both branches see the same
+    latent x_i and thresholds; the Euler step uses the guided velocity."""
+    n_steps, tau_low, tau_high, delta, warmup, method = _loop_args(cfg, n_steps, tau_low, tau_high, delta, warmup,
+                                                                   method)
+    sig = sigmas(n_steps, shift)
+    bc = SamplerBranch(cfg, w, text_cond, tau_low, tau_high, delta, warmup, method, probe_blocks, signal_poly)
+    bu = SamplerBranch(cfg, w, text_uncond, tau_low, tau_high, delta, warmup, method, probe_blocks, signal_poly)
+    x = np.asarray(latent, F64)
+    res = GuidedResult(latent=x)
+    for i in range(n_steps):
+        si = step_inputs(cfg, w, x, 1000.0 * sig[i])
+        tf = _step_override(tau_schedule, i)
+        fc, fu = _step_override(forced_cond, i), _step_override(forced_uncond, i)
+        if force_last and i == n_steps - 1:
+            fc = True if fc is None else fc
+            fu = True if fu is None else fu
+        vc, rc = bc.velocity(i, x, si, fc, tf)
+        vu, ru = bu.velocity(i, x, si, fu, tf)
+        res.cond.append(rc)
+        res.uncond.append(ru)
+        x = euler_step(x, guided_velocity(vc, vu, scale), sig[i], sig[i + 1])
+    res.latent = x
+    return res
+
