@@ -378,6 +378,48 @@ acid_status acid_denoise_loop_graph(const acid_model* m, const acid_loop_cfg* cf
                                     const void* text, acid_step_log* log, void* workspace,
                                     size_t workspace_bytes, acid_stream_t stream);
 
+/* ------------------------------------------------------------------------ */
+/* Classifier-free guidance (the paper is silent on guidance)                 */
+/* ------------------------------------------------------------------------ */
+/* Two branches share the latent: the conditional one (text_cond) and the
+ * unconditional one (text_uncond).  Each branch has its own acid_loop_cfg
+ * (thresholds, forced decisions, method; n_steps and shift must agree), its
+ * own acid_loop_state and its own half of the workspace, so Algorithm 1's
+ * Sigma and s_prev and the base method's cache are kept per branch and the
+ * branches decide independently.  Step i evaluates both branches on x_i
+ * (conditional first) and then x_{i+1} = x_i + (sigma_{i+1} - sigma_i)
+ * (v_u + g (v_c - v_u)), g = guidance_scale.
+ * Workspace: >= acid_guided_workspace_size bytes, 1024-byte aligned; the
+ * unconditional half starts at the first 1024-byte boundary past the
+ * single-branch loop workspace size. */
+acid_status acid_guided_workspace_size(const acid_model* m, size_t* bytes);
+
+/* acid_loop_begin for both branches (texts: device, as acid_loop_begin). */
+acid_status acid_guided_begin(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                              const acid_loop_cfg* cfg_uncond, const void* text_cond,
+                              const void* text_uncond, acid_loop_state* state_cond,
+                              acid_loop_state* state_uncond, void* workspace,
+                              size_t workspace_bytes, acid_stream_t stream);
+
+/* One guided step.  Both states must be at the same step.  log_cond /
+ * log_uncond: host, one entry each, or NULL; ms of the conditional entry is
+ * that branch's time, ms of the unconditional entry covers that branch and
+ * the guided Euler update.  Synchronises once per non-warmup branch step,
+ * as acid_denoise_step does.  guidance_scale must be finite. */
+acid_status acid_guided_step(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                             const acid_loop_cfg* cfg_uncond, double guidance_scale,
+                             acid_loop_state* state_cond, acid_loop_state* state_uncond,
+                             void* latent, acid_step_log* log_cond, acid_step_log* log_uncond,
+                             void* workspace, size_t workspace_bytes, acid_stream_t stream);
+
+/* acid_guided_begin followed by n_steps calls of acid_guided_step.
+ *   log_cond, log_uncond   host [n_steps] each, or NULL. */
+acid_status acid_denoise_loop_guided(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                                     const acid_loop_cfg* cfg_uncond, double guidance_scale,
+                                     void* latent, const void* text_cond, const void* text_uncond,
+                                     acid_step_log* log_cond, acid_step_log* log_uncond,
+                                     void* workspace, size_t workspace_bytes, acid_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -104,6 +104,15 @@ _PROTOS = {
                                     C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
     "acid_denoise_loop_graph": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), _P, _P,
                                           C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
+    "acid_guided_workspace_size": (C.c_int, [C.POINTER(acid_model), C.POINTER(C.c_size_t)]),
+    "acid_guided_begin": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), C.POINTER(acid_loop_cfg), _P, _P,
+                                    C.POINTER(acid_loop_state), C.POINTER(acid_loop_state), _P, C.c_size_t, _P]),
+    "acid_guided_step": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), C.POINTER(acid_loop_cfg),
+                                   C.c_double, C.POINTER(acid_loop_state), C.POINTER(acid_loop_state), _P,
+                                   C.POINTER(acid_step_log), C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
+    "acid_denoise_loop_guided": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), C.POINTER(acid_loop_cfg),
+                                           C.c_double, _P, _P, _P, C.POINTER(acid_step_log),
+                                           C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
 }
 
 _lib = None

@@ -376,3 +376,52 @@ def acid_denoise_loop(model: DeviceModel, cfg_struct, latent: torch.Tensor, text
     check(fn(C.byref(model.struct), C.byref(cfg_struct), latent.data_ptr(), _ptr(text), logs if log else None, ptr,
              nbytes, _stream(stream)))
     return [log_to_dict(x) for x in logs] if log else []
+
+
+# ---------------------------------------------------------------------------
+# classifier-free guidance: two independently cached branches
+# ---------------------------------------------------------------------------
+
+def guided_workspace_size(model: DeviceModel) -> int:
+    b = C.c_size_t()
+    check(load().acid_guided_workspace_size(C.byref(model.struct), C.byref(b)))
+    return b.value
+
+
+class GuidedLoop:
+    """A guided generation driven step by step: acid_guided_begin + acid_guided_step."""
+
+    def __init__(self, model: DeviceModel, cfg_cond, cfg_uncond, scale: float, text_cond, text_uncond,
+                 device="cuda", stream=None):
+        self.model, self.cfg_c, self.cfg_u, self.scale = model, cfg_cond, cfg_uncond, float(scale)
+        self.ws, self.ws_ptr, self.ws_bytes = _aligned_ws(guided_workspace_size(model), device)
+        self.st_c, self.st_u = A.acid_loop_state(), A.acid_loop_state()
+        self.texts = (text_cond, text_uncond)
+        self.stream = stream
+        check(load().acid_guided_begin(C.byref(model.struct), C.byref(cfg_cond), C.byref(cfg_uncond),
+                                       _ptr(text_cond), _ptr(text_uncond), C.byref(self.st_c), C.byref(self.st_u),
+                                       self.ws_ptr, self.ws_bytes, _stream(stream)))
+
+    def step(self, latent: torch.Tensor, log: bool = True):
+        lc, lu = A.acid_step_log(), A.acid_step_log()
+        check(load().acid_guided_step(C.byref(self.model.struct), C.byref(self.cfg_c), C.byref(self.cfg_u),
+                                      self.scale, C.byref(self.st_c), C.byref(self.st_u), latent.data_ptr(),
+                                      C.byref(lc) if log else None, C.byref(lu) if log else None, self.ws_ptr,
+                                      self.ws_bytes, _stream(self.stream)))
+        return (lc, lu) if log else None
+
+
+def acid_denoise_loop_guided(model: DeviceModel, cfg_cond, cfg_uncond, scale: float, latent: torch.Tensor,
+                             text_cond: torch.Tensor | None = None, text_uncond: torch.Tensor | None = None,
+                             log: bool = True, stream=None) -> tuple[list[dict], list[dict]]:
+    """Runs a guided generation in place on latent; returns the two branches' step logs."""
+    _need_cuda(latent, text_cond, text_uncond)
+    if latent.dtype != torch.float32:
+        raise TypeError("latent must be fp32")
+    n = cfg_cond.n_steps
+    lc, lu = (A.acid_step_log * n)(), (A.acid_step_log * n)()
+    ws, ptr, nbytes = _aligned_ws(guided_workspace_size(model), latent.device)
+    check(load().acid_denoise_loop_guided(C.byref(model.struct), C.byref(cfg_cond), C.byref(cfg_uncond), float(scale),
+                                          latent.data_ptr(), _ptr(text_cond), _ptr(text_uncond),
+                                          lc if log else None, lu if log else None, ptr, nbytes, _stream(stream)))
+    return ([log_to_dict(x) for x in lc], [log_to_dict(x) for x in lu]) if log else ([], [])

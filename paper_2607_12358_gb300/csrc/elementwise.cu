@@ -433,6 +433,16 @@ __global__ void euler_kernel(float* lat, const float* __restrict__ v, int64_t n,
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) lat[i] = fmaf(dsig, v[i], lat[i]);
 }
 
+// Classifier-free guidance and the Euler step: x += dsig * (v_u + g (v_c - v_u)).
+__global__ void guided_euler_kernel(float* lat, const float* __restrict__ vc, const float* __restrict__ vu, int64_t n,
+                                    float g, float dsig) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float u = vu[i];
+    lat[i] = fmaf(dsig, fmaf(g, vc[i] - u, u), lat[i]);
+  }
+}
+
 // dsigma = sigma[step + 1] - sigma[step] with the step index read from device memory
 __global__ void euler_sig_kernel(float* lat, const float* __restrict__ v, int64_t n, const double* sig,
                                  const int* step) {
@@ -619,6 +629,13 @@ acid_status unpatchify_euler(const float* vtok, float* v_out, float* latent, int
 
 acid_status euler_update(float* latent, const float* v, int64_t n, float dsigma, cudaStream_t s) {
   euler_kernel<<<grid_for(n), kThreads, 0, s>>>(latent, v, n, dsigma);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status guided_euler_update(float* latent, const float* v_cond, const float* v_uncond, int64_t n, float scale,
+                               float dsigma, cudaStream_t s) {
+  guided_euler_kernel<<<grid_for(n), kThreads, 0, s>>>(latent, v_cond, v_uncond, n, scale, dsigma);
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }

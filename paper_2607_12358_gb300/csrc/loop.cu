@@ -1,12 +1,16 @@
 // The sampling loop of Algorithm 1 (Sec. 3.3) around an Euler flow-matching
-// sampler, with TeaCache or EasyCache (Sec. 2) as the wrapped method.  All
-// tensor work runs in the library's kernels; the host keeps only the scalar
+// sampler, with TeaCache, EasyCache or DiCache (Sec. 2) as the wrapped
+// method, with or without classifier-free guidance.  All tensor work runs in
+// the library's kernels.  The host-driven loop keeps only the scalar
 // controller state and takes one decision per non-warmup step from the drift
-// value it reads back.
+// value it reads back; the graph-launched loop takes it on the device.
 #include <math.h>
 #include <string.h>
 
+#include <cmath>
+
 #include <string>
+#include <utility>
 
 #include "block.h"
 #include "common.cuh"
@@ -411,18 +415,44 @@ extern "C" acid_status acid_loop_begin(const acid_model* m, const acid_loop_cfg*
   return ACID_OK;
 }
 
-extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cfg* cfg, acid_loop_state* st,
-                                         void* latent_v, acid_step_log* log, void* workspace, size_t workspace_bytes,
-                                         acid_stream_t stream) {
-  clear_error();
-  ACID_REQUIRE(m && cfg && st && latent_v, ACID_ERR_INVALID_ARG, "acid_denoise_step: null argument");
-  ACID_TRY(validate_cfg(*cfg));
-  ACID_REQUIRE(st->step >= 0 && st->step < cfg->n_steps, ACID_ERR_INVALID_ARG, "acid_denoise_step: step out of range");
-  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_denoise_step: latent must be 16-byte aligned");
-  LoopWs w;
-  ACID_TRY(check_ws(*m, workspace, workspace_bytes, &w));
-  cudaStream_t s = (cudaStream_t)stream;
-  float* latent = static_cast<float*>(latent_v);
+// CUDA-event timing of one step (only when a log is requested).
+struct StepTimer {
+  bool on;
+  cudaStream_t s;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  StepTimer(bool on_, cudaStream_t s_) : on(on_), s(s_) {}
+  ~StepTimer() {
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+  }
+  acid_status start() {
+    if (!on) return ACID_OK;
+    ACID_CUDA(cudaEventCreate(&e0));
+    ACID_CUDA(cudaEventCreate(&e1));
+    ACID_CUDA(cudaEventRecord(e0, s));
+    return ACID_OK;
+  }
+  // Milliseconds since start (or the previous lap); synchronises on the event.
+  acid_status stop(double* ms) {
+    ACID_CUDA(cudaEventRecord(e1, s));
+    ACID_CUDA(cudaEventSynchronize(e1));
+    float f = 0.f;
+    ACID_CUDA(cudaEventElapsedTime(&f, e0, e1));
+    *ms = f;
+    std::swap(e0, e1);
+    return ACID_OK;
+  }
+};
+
+// One branch's model evaluation at step st->step: Algorithm 1's decision,
+// then the base method's compute or reuse.  defer_euler = false applies the
+// Euler update to the latent in place; defer_euler = true leaves the latent
+// unchanged and points *v_out at the branch's velocity (fp32, latent layout,
+// inside w).  Fills the step log's fields except ms; does not advance
+// st->step.
+static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, acid_loop_state* st, float* latent,
+                               const LoopWs& w, bool defer_euler, const float** v_out, acid_step_log& lg,
+                               cudaStream_t s) {
   const Shape sh = shape_of(*m);
   const int dt = m->block.dtype;
   const int i = st->step;
@@ -432,19 +462,11 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
   const bool warm = i < cfg->warmup;
   int forced = cfg->forced ? cfg->forced[i] : -1;
   if (forced < 0 && cfg->force_last && i == cfg->n_steps - 1) forced = 1;
-
-  acid_step_log lg;
   memset(&lg, 0, sizeof(lg));
   lg.step = i;
   lg.warmup = warm;
   lg.t = t;
   lg.signal = lg.dsignal = lg.tau = lg.sigma = NAN;
-  cudaEvent_t ev0 = nullptr, ev1 = nullptr;
-  if (log) {
-    ACID_CUDA(cudaEventCreate(&ev0));
-    ACID_CUDA(cudaEventCreate(&ev1));
-    ACID_CUDA(cudaEventRecord(ev0, s));
-  }
 
   // timestep embedding: temb = W2 SiLU(W1 sinusoid(t) + b1) + b2
   ACID_TRY(timestep_sinusoid(w.sinus, t, m->time_freq_dim, s));
@@ -491,7 +513,8 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
     } else {
       ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s));
     }
-    ACID_TRY(final_layer(*m, w, x_video, nullptr, latent, dsig, s));
+    ACID_TRY(final_layer(*m, w, x_video, defer_euler ? w.v[0] : nullptr, defer_euler ? nullptr : latent, dsig, s));
+    if (defer_euler) *v_out = w.v[0];
   } else if (cfg->method == ACID_METHOD_DICACHE) {
     // probe: the first probe_blocks blocks on every step; P_i (fp32) in temni[i & 1]
     const int pb = cfg->probe_blocks;
@@ -517,7 +540,8 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
     } else {
       ACID_TRY(dicache_reuse(dt, x_video, p_cur, w, sh.N * sh.d, s));
     }
-    ACID_TRY(final_layer(*m, w, x_video, nullptr, latent, dsig, s));
+    ACID_TRY(final_layer(*m, w, x_video, defer_euler ? w.v[0] : nullptr, defer_euler ? nullptr : latent, dsig, s));
+    if (defer_euler) *v_out = w.v[0];
   } else {
     // EasyCache: s_t = k mean|x_t - x_{t-1}| / mean|v_{t-1}|
     float* v = w.v[i & 1];
@@ -553,18 +577,33 @@ extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cf
       ACID_TRY(add_mixed(ACID_FP32, latent, ACID_FP32, w.offset, ACID_FP32, v, sh.latent, 1.0f, s));
     }
     ACID_CUDA(cudaMemcpyAsync(w.x_prev, latent, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
-    ACID_TRY(euler_update(latent, v, sh.latent, dsig, s));
+    if (defer_euler)
+      *v_out = v;
+    else
+      ACID_TRY(euler_update(latent, v, sh.latent, dsig, s));
   }
   lg.computed = compute;
-  st->step = i + 1;
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_denoise_step(const acid_model* m, const acid_loop_cfg* cfg, acid_loop_state* st,
+                                         void* latent_v, acid_step_log* log, void* workspace, size_t workspace_bytes,
+                                         acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m && cfg && st && latent_v, ACID_ERR_INVALID_ARG, "acid_denoise_step: null argument");
+  ACID_TRY(validate_cfg(*cfg));
+  ACID_REQUIRE(st->step >= 0 && st->step < cfg->n_steps, ACID_ERR_INVALID_ARG, "acid_denoise_step: step out of range");
+  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_denoise_step: latent must be 16-byte aligned");
+  LoopWs w;
+  ACID_TRY(check_ws(*m, workspace, workspace_bytes, &w));
+  cudaStream_t s = (cudaStream_t)stream;
+  StepTimer tm(log != nullptr, s);
+  ACID_TRY(tm.start());
+  acid_step_log lg;
+  ACID_TRY(branch_step(m, cfg, st, static_cast<float*>(latent_v), w, false, nullptr, lg, s));
+  st->step += 1;
   if (log) {
-    ACID_CUDA(cudaEventRecord(ev1, s));
-    ACID_CUDA(cudaEventSynchronize(ev1));
-    float ms = 0.f;
-    ACID_CUDA(cudaEventElapsedTime(&ms, ev0, ev1));
-    lg.ms = ms;
-    cudaEventDestroy(ev0);
-    cudaEventDestroy(ev1);
+    ACID_TRY(tm.stop(&lg.ms));
     *log = lg;
   }
   return ACID_OK;
@@ -577,6 +616,106 @@ extern "C" acid_status acid_denoise_loop(const acid_model* m, const acid_loop_cf
   ACID_TRY(acid_loop_begin(m, cfg, text, &st, workspace, workspace_bytes, stream));
   for (int i = 0; i < cfg->n_steps; ++i)
     ACID_TRY(acid_denoise_step(m, cfg, &st, latent, log ? log + i : nullptr, workspace, workspace_bytes, stream));
+  return ACID_OK;
+}
+
+// ===========================================================================
+// Classifier-free guidance: two branches (conditional and unconditional
+// text), each with its own loop workspace, Algorithm 1 state and cache; the
+// Euler step takes v = v_u + g (v_c - v_u).
+// ===========================================================================
+
+static size_t guided_half(const acid_model& m) { return (loop_layout(m, nullptr).bytes + 1023) / 1024 * 1024; }
+
+static acid_status guided_check(const acid_model* m, const acid_loop_cfg* cc, const acid_loop_cfg* cu, void* ws,
+                                size_t bytes, LoopWs* wc, LoopWs* wu) {
+  ACID_REQUIRE(m && cc && cu, ACID_ERR_INVALID_ARG, "guided loop: null argument");
+  ACID_TRY(validate_cfg(*cc));
+  ACID_TRY(validate_cfg(*cu));
+  ACID_REQUIRE(cc->n_steps == cu->n_steps && cc->shift == cu->shift, ACID_ERR_INVALID_ARG,
+               "guided loop: both branches need the same n_steps and shift");
+  ACID_REQUIRE(ws != nullptr && aligned(ws, 1024), ACID_ERR_WORKSPACE,
+               "guided loop: workspace null or not 1024-aligned");
+  const size_t half = guided_half(*m);
+  ACID_REQUIRE(bytes >= 2 * half, ACID_ERR_WORKSPACE,
+               "guided loop: workspace too small (need " + std::to_string(2 * half) + " bytes)");
+  *wc = loop_layout(*m, ws);
+  *wu = loop_layout(*m, static_cast<uint8_t*>(ws) + half);
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_guided_workspace_size(const acid_model* m, size_t* bytes) {
+  clear_error();
+  ACID_REQUIRE(m && bytes, ACID_ERR_INVALID_ARG, "acid_guided_workspace_size: null argument");
+  ACID_TRY(validate_model(*m));
+  *bytes = 2 * guided_half(*m);
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_guided_begin(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                                         const acid_loop_cfg* cfg_uncond, const void* text_cond,
+                                         const void* text_uncond, acid_loop_state* state_cond,
+                                         acid_loop_state* state_uncond, void* workspace, size_t workspace_bytes,
+                                         acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m, ACID_ERR_INVALID_ARG, "acid_guided_begin: null model");
+  ACID_TRY(validate_model(*m));
+  LoopWs wc, wu;
+  ACID_TRY(guided_check(m, cfg_cond, cfg_uncond, workspace, workspace_bytes, &wc, &wu));
+  const size_t half = guided_half(*m);
+  ACID_TRY(acid_loop_begin(m, cfg_cond, text_cond, state_cond, workspace, half, stream));
+  ACID_TRY(acid_loop_begin(m, cfg_uncond, text_uncond, state_uncond, static_cast<uint8_t*>(workspace) + half, half,
+                           stream));
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_guided_step(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                                        const acid_loop_cfg* cfg_uncond, double guidance_scale,
+                                        acid_loop_state* state_cond, acid_loop_state* state_uncond, void* latent_v,
+                                        acid_step_log* log_cond, acid_step_log* log_uncond, void* workspace,
+                                        size_t workspace_bytes, acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(state_cond && state_uncond && latent_v, ACID_ERR_INVALID_ARG, "acid_guided_step: null argument");
+  LoopWs wc, wu;
+  ACID_TRY(guided_check(m, cfg_cond, cfg_uncond, workspace, workspace_bytes, &wc, &wu));
+  ACID_REQUIRE(state_cond->step == state_uncond->step && state_cond->step >= 0 &&
+                   state_cond->step < cfg_cond->n_steps,
+               ACID_ERR_INVALID_ARG, "acid_guided_step: branch steps differ or out of range");
+  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_guided_step: latent must be 16-byte aligned");
+  ACID_REQUIRE(std::isfinite(guidance_scale), ACID_ERR_INVALID_ARG, "acid_guided_step: guidance scale not finite");
+  cudaStream_t s = (cudaStream_t)stream;
+  float* latent = static_cast<float*>(latent_v);
+  const int i = state_cond->step;
+  const float dsig = (float)(sigma_at(*cfg_cond, i + 1) - sigma_at(*cfg_cond, i));
+  const bool timed = log_cond || log_uncond;
+  StepTimer tm(timed, s);
+  ACID_TRY(tm.start());
+  acid_step_log lc, lu;
+  const float *vc = nullptr, *vu = nullptr;
+  ACID_TRY(branch_step(m, cfg_cond, state_cond, latent, wc, true, &vc, lc, s));
+  if (timed) ACID_TRY(tm.stop(&lc.ms));
+  ACID_TRY(branch_step(m, cfg_uncond, state_uncond, latent, wu, true, &vu, lu, s));
+  ACID_TRY(guided_euler_update(latent, vc, vu, shape_of(*m).latent, (float)guidance_scale, dsig, s));
+  if (timed) ACID_TRY(tm.stop(&lu.ms));
+  state_cond->step += 1;
+  state_uncond->step += 1;
+  if (log_cond) *log_cond = lc;
+  if (log_uncond) *log_uncond = lu;
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_denoise_loop_guided(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                                                const acid_loop_cfg* cfg_uncond, double guidance_scale,
+                                                void* latent, const void* text_cond, const void* text_uncond,
+                                                acid_step_log* log_cond, acid_step_log* log_uncond, void* workspace,
+                                                size_t workspace_bytes, acid_stream_t stream) {
+  acid_loop_state sc, su;
+  ACID_TRY(acid_guided_begin(m, cfg_cond, cfg_uncond, text_cond, text_uncond, &sc, &su, workspace, workspace_bytes,
+                             stream));
+  for (int i = 0; i < cfg_cond->n_steps; ++i)
+    ACID_TRY(acid_guided_step(m, cfg_cond, cfg_uncond, guidance_scale, &sc, &su, latent,
+                              log_cond ? log_cond + i : nullptr, log_uncond ? log_uncond + i : nullptr, workspace,
+                              workspace_bytes, stream));
   return ACID_OK;
 }
 
