@@ -23,6 +23,8 @@
 #include <cudaTypedefs.h>
 #include <math.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -148,15 +150,21 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (lane == 0) {  // ---------------------------------------- MMA issuer
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, kBKV, false, false);
       constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
-      const uint32_t q0 = smem_u32(sQ);
+      // Shared-memory descriptors are built once; an operand at byte offset o
+      // from a base is the base descriptor plus o >> 4 (the 14-bit address
+      // field cannot overflow: shared memory ends below 256 KB).
+      const uint64_t qdesc = smem_desc_sw128(smem_u32(sQ), 16, 1024);
+      const uint64_t kdesc = smem_desc_sw128(smem_u32(sK), 16, 1024);
+      const uint64_t vdesc = smem_desc_sw128(smem_u32(sV), C::CHUNK_BYTES, 1024);
       // S_t(j) = Q_t K_j^T into the S region of tile t
       auto issue_s = [&](int t, int j) {
-        const uint32_t k0 = smem_u32(sK + (j & 1) * C::T_BYTES);
+        const uint64_t a0 = qdesc + (uint64_t)((t * C::T_BYTES) >> 4);
+        const uint64_t b0 = kdesc + (uint64_t)(((j & 1) * C::T_BYTES) >> 4);
+        const uint32_t d = tmem + C::S_COL + t * kBKV;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
-          mma_bf16_ss(tmem + C::S_COL + t * kBKV, smem_desc_sw128(q0 + t * C::T_BYTES + off, 16, 1024),
-                      smem_desc_sw128(k0 + off, 16, 1024), idesc_s, kk != 0);
+          const uint64_t off = (uint64_t)(((kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32) >> 4);
+          mma_bf16_ss(d, a0 + off, b0 + off, idesc_s, kk != 0);
         }
         mma_commit(&s_full[t]);
       };
@@ -174,11 +182,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           if (t == 0 && !mbar_wait(&v_full[st], (j >> 1) & 1)) { ok = false; break; }
           tc_fence_after();
           // O_t += P_t V_j: P_t (128 x 128 keys) from TMEM, V_j MN-major from shared memory
-          const uint32_t v0 = smem_u32(sV + st * C::T_BYTES);
+          const uint64_t b0 = vdesc + (uint64_t)((st * C::T_BYTES) >> 4);
+          const uint32_t d = tmem + C::O_COL + t * 128, p0 = tmem + C::S_COL + t * kBKV;
 #pragma unroll
           for (int kk = 0; kk < kBKV / 16; ++kk)
-            mma_bf16_ts(tmem + C::O_COL + t * 128, tmem + C::S_COL + t * kBKV + kk * 8,
-                        smem_desc_sw128(v0 + kk * 16 * 128, C::CHUNK_BYTES, 1024), idesc_o, (j | kk) != 0);
+            mma_bf16_ts(d, p0 + kk * 8, b0 + (uint64_t)((kk * 16 * 128) >> 4), idesc_o, (j | kk) != 0);
           mma_commit(&pv_done[t]);
           if (t == 1) mma_commit(&v_empty[st]);
           if (j + 1 < nkv) {
@@ -199,58 +207,64 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const uint32_t o_addr = tmem + lane_base + C::O_COL + t * 128;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int j = 0; j < nkv; ++j) {
-      if (!mbar_wait(&s_full[t], j & 1)) { ok = false; break; }
+    // One key tile; the masked variant (keys past the end of the sequence)
+    // is compiled separately and runs only on a partial last tile.
+    auto step = [&](int j, auto masked) -> bool {
+      if (!mbar_wait(&s_full[t], j & 1)) return false;
       // consume pv_done_t phase j-1 (already complete: s_full_t(j) is committed
       // after PV_t(j-1)) so that the final parity wait is never two phases ahead
-      if (j > 0 && !mbar_wait(&pv_done[t], (j - 1) & 1)) { ok = false; break; }
+      if (j > 0 && !mbar_wait(&pv_done[t], (j - 1) & 1)) return false;
       tc_fence_after();
       float s[kBKV];
 #pragma unroll
       for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
       tmem_wait_ld();
-      const int64_t kv0 = (int64_t)(jb + j) * kBKV;
-      if (kv0 + kBKV > a.nk) {
-#pragma unroll
-        for (int i = 0; i < kBKV; ++i)
-          if (kv0 + i >= a.nk) s[i] = -INFINITY;
-      }
-      // row max of the raw scores (four independent 3-input max chains); the
-      // positive scale commutes with max, so it is applied to the max only
-      float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-      for (int i = 0; i < kBKV; i += 8) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) m4[k] = fmax3(m4[k], s[i + 2 * k], s[i + 2 * k + 1]);
-      }
-      const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * a.scale_log2;
-      // s_full_t(j) is committed after PV_t(j-1), so O_t and the P_t region are
-      // free here.  Lazy rescaling: keep the reference max unless it grew by 2^8.
       bool resc = false;
       float f = 1.0f;
-      if (j > 0) {
-        resc = mx > m_run + kRescaleLog2;
-        if (resc) {
-          f = ex2_approx(m_run - mx);
-          l_run *= f;
-          m_run = mx;
-        }
-      } else {
-        m_run = mx;
+      if constexpr (decltype(masked)::value) {
+        const int valid = (int)(a.nk - (int64_t)(jb + j) * kBKV);  // keys of the last tile
+#pragma unroll
+        for (int i = 0; i < kBKV; ++i)
+          if (i >= valid) s[i] = -INFINITY;
       }
-      // P = 2^(s * scale - m_run) as bf16 pairs over the first 64 columns of S_t;
-      // the scale-and-subtract and the row sum run as packed fp32 pairs
+      // e = s * scale - m_run in place (packed pairs; the first tile uses 0 as
+      // the reference), with the row max of e alongside in four independent
+      // 3-input max chains on the ALU pipe.  s_full_t(j) is committed after
+      // PV_t(j-1), so O_t and the P_t region are free here.  Lazy rescaling:
+      // the reference max moves only on the first tile or when the row max
+      // exceeds it by more than 2^8; then e is shifted in place.
       const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2);
-      const uint64_t nm2 = f2_pack(-m_run, -m_run);
+      {
+        const float mref = j == 0 ? 0.f : m_run;
+        const uint64_t nm2 = f2_pack(-mref, -mref);
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+        for (int i = 0; i < kBKV / 2; ++i) {
+          f2_unpack(f2_fma(f2_pack(s[2 * i], s[2 * i + 1]), sc2, nm2), s[2 * i], s[2 * i + 1]);
+          m4[i & 3] = fmax3(m4[i & 3], s[2 * i], s[2 * i + 1]);
+        }
+        const float me = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        if (j == 0 || me > kRescaleLog2) {
+          if (j > 0) {
+            resc = true;
+            f = ex2_approx(-me);
+            l_run *= f;
+          }
+          m_run = mref + me;
+          const uint64_t sh2 = f2_pack(-me, -me);
+#pragma unroll
+          for (int i = 0; i < kBKV / 2; ++i) f2_unpack(f2_add(f2_pack(s[2 * i], s[2 * i + 1]), sh2), s[2 * i], s[2 * i + 1]);
+        }
+      }
+      // P = 2^e as bf16 pairs over the first 64 columns of S_t, with the row
+      // sum as packed fp32 pairs
       uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t pk[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          float e0, e1;
-          f2_unpack(f2_fma(f2_pack(s[half * 64 + 2 * i], s[half * 64 + 2 * i + 1]), sc2, nm2), e0, e1);
-          const float p0 = ex2_approx(e0), p1 = ex2_approx(e1);
+          const float p0 = ex2_approx(s[half * 64 + 2 * i]), p1 = ex2_approx(s[half * 64 + 2 * i + 1]);
           if (i & 1)
             acc1 = f2_add(acc1, f2_pack(p0, p1));
           else
@@ -278,6 +292,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       tmem_wait_st();
       tc_fence_before();
       mbar_arrive(&p_full[t]);
+          return true;
+    };
+    const bool partial_last = (int64_t)(jb + nkv) * kBKV > a.nk;
+    for (int j = 0; j < nkv; ++j) {
+      const bool ok_j = (j == nkv - 1 && partial_last) ? step(j, std::true_type{}) : step(j, std::false_type{});
+      if (!ok_j) {
+        ok = false;
+        break;
+      }
     }
     // ---------------------------------------------------- epilogue: O_t / l
     if (ok) ok = mbar_wait(&pv_done[t], (nkv - 1) & 1);
