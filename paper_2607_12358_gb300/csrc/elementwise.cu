@@ -594,6 +594,10 @@ RopeTable rope_layout(int grid_f, int grid_h, int grid_w, int head_dim) {
   const int dt = head_dim - 2 * dh;
   t.grid_f = grid_f; t.grid_h = grid_h; t.grid_w = grid_w;
   t.pairs_t = dt / 2; t.pairs_h = dh / 2; t.pairs_w = dh / 2;
+  if (grid_h > 0 && grid_w > 0) {
+    t.inv_hw = 1.0f / (float)(grid_h * grid_w);
+    t.inv_w = 1.0f / (float)grid_w;
+  }
   return t;
 }
 

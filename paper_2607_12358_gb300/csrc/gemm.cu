@@ -56,19 +56,38 @@ EpiDev to_dev(const Epilogue& e) {
   return d;
 }
 
-// (cos, sin) of the RoPE angle of pair `jj` (within the head) at video position pos.
-__device__ __forceinline__ float2 rope_cs(const RopeTable& t, int64_t pos, int jj) {
-  const int64_t hw = (int64_t)t.grid_h * t.grid_w;
-  const int f = (int)(pos / hw);
-  const int h = (int)((pos / t.grid_w) % t.grid_h);
-  const int w = (int)(pos % t.grid_w);
-  if (jj < t.pairs_t) return t.table[(int64_t)f * t.pairs_t + jj];
+// Video position -> (frame, row, column) of the latent grid in 32-bit
+// arithmetic.  Positions are below 2^24 (checked on the host), so the float
+// quotient n * (1/d) is within one of floor(n / d) and one correction step
+// makes it exact.
+struct RopePos {
+  int f, h, w;
+};
+__device__ __forceinline__ int div_small(int n, int d, float inv_d) {
+  int q = (int)((float)n * inv_d);
+  const int r = n - q * d;
+  q += (r >= d) - (r < 0);
+  return q;
+}
+__device__ __forceinline__ RopePos rope_pos(const RopeTable& t, int pos) {
+  const int hw = t.grid_h * t.grid_w;
+  RopePos p;
+  p.f = div_small(pos, hw, t.inv_hw);
+  const int rem = pos - p.f * hw;
+  p.h = div_small(rem, t.grid_w, t.inv_w);
+  p.w = rem - p.h * t.grid_w;
+  return p;
+}
+
+// (cos, sin) of the RoPE angle of pair `jj` (within the head) at a decomposed position.
+__device__ __forceinline__ float2 rope_cs(const RopeTable& t, const RopePos& p, int jj) {
+  if (jj < t.pairs_t) return t.table[p.f * t.pairs_t + jj];
   jj -= t.pairs_t;
-  const int64_t off_h = (int64_t)t.grid_f * t.pairs_t;
-  if (jj < t.pairs_h) return t.table[off_h + (int64_t)h * t.pairs_h + jj];
+  const int off_h = t.grid_f * t.pairs_t;
+  if (jj < t.pairs_h) return t.table[off_h + p.h * t.pairs_h + jj];
   jj -= t.pairs_h;
-  const int64_t off_w = off_h + (int64_t)t.grid_h * t.pairs_h;
-  return t.table[off_w + (int64_t)w * t.pairs_w + jj];
+  const int off_w = off_h + t.grid_h * t.pairs_h;
+  return t.table[off_w + p.w * t.pairs_w + jj];
 }
 
 // Applies the epilogue to the adjacent outputs (grow, col) and (grow, col+1).
@@ -87,7 +106,7 @@ __device__ __forceinline__ void epi_pair(const EpiDev& e, int64_t grow, int col,
       break;
     case EPI_ROPE_QKV:
       if (col < 2 * e.d && grow >= e.rope_first_video) {
-        const float2 cs = rope_cs(e.rope, grow - e.rope_first_video, (col % e.head_dim) >> 1);
+        const float2 cs = rope_cs(e.rope, rope_pos(e.rope, (int)(grow - e.rope_first_video)), (col % e.head_dim) >> 1);
         const float x0 = a, x1 = b;
         a = x0 * cs.x - x1 * cs.y;
         b = x0 * cs.y + x1 * cs.x;
@@ -201,9 +220,13 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
         break;
       case EPI_ROPE_QKV:
         if (col < 2 * e.d && grow >= e.rope_first_video) {
+          // one position decomposition per row; the four columns lie in one
+          // head (head_dim is a power of two, checked on the host)
+          const RopePos pp = rope_pos(e.rope, (int)(grow - e.rope_first_video));
+          const int j0 = (col & (e.head_dim - 1)) >> 1;
 #pragma unroll
           for (int k = 0; k < 4; k += 2) {
-            const float2 cs = rope_cs(e.rope, grow - e.rope_first_video, ((col + k) % e.head_dim) >> 1);
+            const float2 cs = rope_cs(e.rope, pp, j0 + (k >> 1));
             const float x0 = v[k], x1 = v[k + 1];
             v[k] = x0 * cs.x - x1 * cs.y;
             v[k + 1] = x0 * cs.y + x1 * cs.x;
@@ -531,12 +554,17 @@ acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int
   if (M == 0) return ACID_OK;
   ACID_REQUIRE(epi.kind != EPI_ROPE_QKV || (epi.rope.table != nullptr && epi.head_dim > 0 && epi.d > 0),
                ACID_ERR_INVALID_ARG, "linear: RoPE epilogue needs a table");
+  ACID_REQUIRE(epi.kind != EPI_ROPE_QKV ||
+                   (int64_t)epi.rope.grid_f * epi.rope.grid_h * epi.rope.grid_w < (int64_t(1) << 24),
+               ACID_ERR_UNSUPPORTED, "linear: RoPE positions must be below 2^24");
   ACID_REQUIRE(!epi_reads_res(epi.kind) || epi.residual != nullptr, ACID_ERR_INVALID_ARG,
                "linear: residual epilogue needs a residual");
   if (dtype == ACID_FP32) return linear_forward_f32(A, lda, M, K, ACID_FP32, W, N, out, ldo, epi, s);
   ACID_REQUIRE(N % 32 == 0 && K % 8 == 0, ACID_ERR_UNSUPPORTED, "linear bf16: need N % 32 == 0 and K % 8 == 0");
   ACID_REQUIRE(ldo % 8 == 0 && aligned(out, 16) && (!epi.residual || (epi.ldr % 8 == 0 && aligned(epi.residual, 16))),
                ACID_ERR_UNSUPPORTED, "linear bf16: output/residual must be 16-byte aligned rows");
+  ACID_REQUIRE(epi.kind != EPI_ROPE_QKV || (epi.head_dim & (epi.head_dim - 1)) == 0, ACID_ERR_UNSUPPORTED,
+               "linear bf16: the RoPE epilogue needs a power-of-two head_dim");
   if (N % 256 == 0) return launch_tc<256>(A, lda, M, K, W, N, out, ldo, epi, s);
   if (N % 128 == 0) return launch_tc<128>(A, lda, M, K, W, N, out, ldo, epi, s);
   return launch_tc<64>(A, lda, M, K, W, N, out, ldo, epi, s);

@@ -16,6 +16,7 @@ struct RopeTable {
   const float2* table = nullptr;  // [F*pt2 | H*ph2 | W*pw2]
   int grid_f = 0, grid_h = 0, grid_w = 0;
   int pairs_t = 0, pairs_h = 0, pairs_w = 0;
+  float inv_hw = 0.f, inv_w = 0.f;  // 1 / (grid_h * grid_w), 1 / grid_w (position decomposition)
   int64_t elems() const {
     return (int64_t)grid_f * pairs_t + (int64_t)grid_h * pairs_h + (int64_t)grid_w * pairs_w;
   }
