@@ -186,36 +186,67 @@ __global__ void add_mixed_kernel(const TA* __restrict__ a, const TB* __restrict_
 // One warp per row; row kept in registers (d <= 256 * kMaxV).
 constexpr int kLnMaxV = 12;
 
-template <typename Tin, typename Tout>
+// NV: 8-element vectors per lane (d <= 256 * NV); sized to the row so that
+// short rows keep few registers and many rows in flight.  The row stays in
+// registers as loaded (bf16 packed, four registers per 8 values) and is
+// unpacked in each of the three passes.
+template <typename Tin, typename Tout, int NV>
 __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict__ x, Tout* __restrict__ y,
                                                           int64_t rows, int d, const float* __restrict__ shv,
                                                           const float* __restrict__ scv,
                                                           const float* __restrict__ sht,
                                                           const float* __restrict__ sct, int64_t split, float eps) {
+  constexpr int kW = sizeof(Tin) == 2 ? 1 : 2;  // uint4 words per 8 values
   const int64_t row = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
   const Tin* xr = x + row * d;
-  float v[kLnMaxV][8];
+  uint4 raw[NV][kW];
+  auto unpack = [&](int i, float* f) {
+    if constexpr (kW == 1) {
+      const uint32_t w[4] = {raw[i][0].x, raw[i][0].y, raw[i][0].z, raw[i][0].w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        f[2 * j] = bf16_lo(w[j]);
+        f[2 * j + 1] = bf16_hi(w[j]);
+      }
+    } else {
+      const float4 p0 = *reinterpret_cast<const float4*>(&raw[i][0]), p1 = *reinterpret_cast<const float4*>(&raw[i][1]);
+      f[0] = p0.x; f[1] = p0.y; f[2] = p0.z; f[3] = p0.w;
+      f[4] = p1.x; f[5] = p1.y; f[6] = p1.z; f[7] = p1.w;
+    }
+  };
   float s = 0.f;
 #pragma unroll
-  for (int i = 0; i < kLnMaxV; ++i) {
+  for (int i = 0; i < NV; ++i) {
     const int c = (i * 32 + lane) * 8;
     if (c < d) {
-      load8(xr + c, v[i]);
+      const uint4* src = reinterpret_cast<const uint4*>(xr + c);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) s += v[i][j];
+      for (int k = 0; k < kW; ++k) raw[i][k] = src[k];
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = (i * 32 + lane) * 8;
+    if (c < d) {
+      float f[8];
+      unpack(i, f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s += f[j];
     }
   }
   const float mean = warp_sum_f(s) / d;
   float q = 0.f;
 #pragma unroll
-  for (int i = 0; i < kLnMaxV; ++i) {
+  for (int i = 0; i < NV; ++i) {
     const int c = (i * 32 + lane) * 8;
     if (c < d) {
+      float f[8];
+      unpack(i, f);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        const float t = v[i][j] - mean;
+        const float t = f[j] - mean;
         q += t * t;
       }
     }
@@ -226,19 +257,20 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
   const float* sc = text ? sct : scv;
   Tout* yr = y + row * d;
 #pragma unroll
-  for (int i = 0; i < kLnMaxV; ++i) {
+  for (int i = 0; i < NV; ++i) {
     const int c = (i * 32 + lane) * 8;
     if (c < d) {
-      float o[8];
+      float f[8], o[8];
+      unpack(i, f);
       if (sc != nullptr) {
         float a[8], b[8];
         load8(sc + c, a);
         load8(sh + c, b);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = fmaf((v[i][j] - mean) * rstd, 1.0f + a[j], b[j]);
+        for (int j = 0; j < 8; ++j) o[j] = fmaf((f[j] - mean) * rstd, 1.0f + a[j], b[j]);
       } else {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = (v[i][j] - mean) * rstd;
+        for (int j = 0; j < 8; ++j) o[j] = (f[j] - mean) * rstd;
       }
       store8(yr + c, o);
     }
@@ -532,24 +564,36 @@ acid_status add_mixed(int ad, const void* a, int bd, const void* b, int od, void
   return ACID_OK;
 }
 
+template <int NV>
+acid_status launch_ln_mod(int in_dtype, int out_dtype, const void* x, void* y, int64_t rows, int d, const float* shv,
+                          const float* scv, const float* sht, const float* sct, int64_t split, float eps, int blocks,
+                          cudaStream_t s) {
+  using H = __nv_bfloat16;
+  if (in_dtype == ACID_BF16 && out_dtype == ACID_BF16)
+    ln_mod_kernel<H, H, NV><<<blocks, kThreads, 0, s>>>((const H*)x, (H*)y, rows, d, shv, scv, sht, sct, split, eps);
+  else if (in_dtype == ACID_BF16)
+    ln_mod_kernel<H, float, NV><<<blocks, kThreads, 0, s>>>((const H*)x, (float*)y, rows, d, shv, scv, sht, sct, split,
+                                                          eps);
+  else if (out_dtype == ACID_BF16)
+    ln_mod_kernel<float, H, NV><<<blocks, kThreads, 0, s>>>((const float*)x, (H*)y, rows, d, shv, scv, sht, sct, split,
+                                                          eps);
+  else
+    ln_mod_kernel<float, float, NV><<<blocks, kThreads, 0, s>>>((const float*)x, (float*)y, rows, d, shv, scv, sht, sct,
+                                                              split, eps);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
 acid_status ln_mod(int in_dtype, const void* x, int out_dtype, void* y, int64_t rows, int d, const float* shv,
                    const float* scv, const float* sht, const float* sct, int64_t split, float eps, cudaStream_t s) {
   ACID_REQUIRE(d % 8 == 0 && d <= 256 * kLnMaxV, ACID_ERR_UNSUPPORTED, "ln_mod: d must be a multiple of 8, <= 3072");
   if (rows == 0) return ACID_OK;
   if (sht == nullptr) { sht = shv; sct = scv; }
   const int64_t blocks = (rows * 32 + kThreads - 1) / kThreads;
-  using H = __nv_bfloat16;
-  if (in_dtype == ACID_BF16 && out_dtype == ACID_BF16)
-    ln_mod_kernel<H, H><<<blocks, kThreads, 0, s>>>((const H*)x, (H*)y, rows, d, shv, scv, sht, sct, split, eps);
-  else if (in_dtype == ACID_BF16)
-    ln_mod_kernel<H, float><<<blocks, kThreads, 0, s>>>((const H*)x, (float*)y, rows, d, shv, scv, sht, sct, split, eps);
-  else if (out_dtype == ACID_BF16)
-    ln_mod_kernel<float, H><<<blocks, kThreads, 0, s>>>((const float*)x, (H*)y, rows, d, shv, scv, sht, sct, split, eps);
-  else
-    ln_mod_kernel<float, float><<<blocks, kThreads, 0, s>>>((const float*)x, (float*)y, rows, d, shv, scv, sht, sct,
-                                                           split, eps);
-  ACID_CHECK_LAUNCH();
-  return ACID_OK;
+  if (d <= 256 * 4) return launch_ln_mod<4>(in_dtype, out_dtype, x, y, rows, d, shv, scv, sht, sct, split, eps, blocks, s);
+  if (d <= 256 * 6) return launch_ln_mod<6>(in_dtype, out_dtype, x, y, rows, d, shv, scv, sht, sct, split, eps, blocks, s);
+  if (d <= 256 * 8) return launch_ln_mod<8>(in_dtype, out_dtype, x, y, rows, d, shv, scv, sht, sct, split, eps, blocks, s);
+  return launch_ln_mod<kLnMaxV>(in_dtype, out_dtype, x, y, rows, d, shv, scv, sht, sct, split, eps, blocks, s);
 }
 
 acid_status ln_mod_drift(const float* x, float* tem0, float* tem1, const int* step_dev, int step_host, int64_t rows,

@@ -79,8 +79,9 @@ __device__ __forceinline__ RopePos rope_pos(const RopeTable& t, int pos) {
   return p;
 }
 
-// (cos, sin) of the RoPE angle of pair `jj` (within the head) at a decomposed position.
-__device__ __forceinline__ float2 rope_cs(const RopeTable& t, const RopePos& p, int jj) {
+// Table entry (cos, sin) of the RoPE angle of pair `jj` (within the head) at a
+// decomposed position.
+__device__ __forceinline__ const float2& rope_cs_ptr(const RopeTable& t, const RopePos& p, int jj) {
   if (jj < t.pairs_t) return t.table[p.f * t.pairs_t + jj];
   jj -= t.pairs_t;
   const int off_h = t.grid_f * t.pairs_t;
@@ -89,6 +90,7 @@ __device__ __forceinline__ float2 rope_cs(const RopeTable& t, const RopePos& p, 
   const int off_w = off_h + t.grid_h * t.pairs_h;
   return t.table[off_w + p.w * t.pairs_w + jj];
 }
+__device__ __forceinline__ float2 rope_cs(const RopeTable& t, const RopePos& p, int jj) { return rope_cs_ptr(t, p, jj); }
 
 // Applies the epilogue to the adjacent outputs (grow, col) and (grow, col+1).
 // r0/r1: residual values (read by the caller) for the residual kinds.
@@ -167,42 +169,79 @@ struct GemmDims {
 // handles columns 4(l%8) .. 4(l%8)+3 of rows 4p + l/8, p = 0..7.  Residual
 // values of the next chunk are loaded while the current one is processed, so
 // each lane keeps up to 16 loads in flight.
+// R32: the residual is fp32 (else bf16); fixed per kernel so that a bf16
+// residual keeps two registers per row
+template <bool R32>
 struct ResChunk {
-  float v[8][4];
+  uint32_t w[8][R32 ? 4 : 2];  // residual of this lane's 4 columns on its 8 rows (bf16 pairs or fp32)
+  float bias[4], gv[4], gt[4];  // per-column bias and gates (video / text stream)
 };
 
-__device__ __forceinline__ void load_res_chunk(const GemmDims& g, const EpiDev& e, int64_t row0, int col,
-                                               ResChunk& rc) {
+// Loads what the epilogue of the chunk at columns [col, col+4) needs from
+// global memory: the residual (for the residual kinds) and the per-column
+// bias and gates, through the read-only path for the vectors.  Called one
+// chunk ahead so that the loads overlap the previous chunk's work.
+template <int KIND, bool R32>
+__device__ __forceinline__ void load_chunk_inputs(const GemmDims& g, const EpiDev& e, int64_t row0, int col,
+                                                  ResChunk<R32>& rc) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int p = 0; p < 8; ++p) {
-    const int64_t row = row0 + 4 * p + (lane >> 3);
-    if (row >= g.M) continue;
-    if (e.res_fp32) {
-      const float4 t = *reinterpret_cast<const float4*>(static_cast<const float*>(e.res) + row * e.ldr + col);
-      rc.v[p][0] = t.x; rc.v[p][1] = t.y; rc.v[p][2] = t.z; rc.v[p][3] = t.w;
-    } else {
-      const uint2 t = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col);
-      rc.v[p][0] = bf16_lo(t.x); rc.v[p][1] = bf16_hi(t.x); rc.v[p][2] = bf16_lo(t.y); rc.v[p][3] = bf16_hi(t.y);
+  for (int k = 0; k < 4; ++k) {
+    rc.bias[k] = e.bias ? __ldg(e.bias + col + k) : 0.f;
+    rc.gv[k] = KIND == EPI_GATED_RES ? __ldg(e.gate_v + col + k) : 0.f;
+    rc.gt[k] = KIND == EPI_GATED_RES ? __ldg(e.gate_t + col + k) : 0.f;
+  }
+  if constexpr (KIND == EPI_GATED_RES || KIND == EPI_RES) {
+#pragma unroll
+    for (int p = 0; p < 8; ++p) {
+      const int64_t row = row0 + 4 * p + (lane >> 3);
+      if (row >= g.M) continue;
+      if constexpr (R32) {
+        const uint4 t = *reinterpret_cast<const uint4*>(static_cast<const float*>(e.res) + row * e.ldr + col);
+        rc.w[p][0] = t.x; rc.w[p][1] = t.y; rc.w[p][2] = t.z; rc.w[p][3] = t.w;
+      } else {
+        const uint2 t = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col);
+        rc.w[p][0] = t.x; rc.w[p][1] = t.y;
+      }
     }
   }
 }
 
-template <int KIND>
+template <bool R32>
+__device__ __forceinline__ float res_value(const ResChunk<R32>& rc, int p, int k) {
+  if constexpr (R32) {
+    return __uint_as_float(rc.w[p][k]);
+  } else {
+    const uint32_t w = rc.w[p][k >> 1];
+    return (k & 1) ? bf16_hi(w) : bf16_lo(w);
+  }
+}
+
+template <int KIND, bool R32>
 __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, float* stage, int64_t row0,
-                                               int col0, const uint32_t* r, const ResChunk& rc) {
+                                               int col0, const uint32_t* r, const ResChunk<R32>& rc) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
   for (int j = 0; j < 32; ++j) stage[lane * 33 + j] = __uint_as_float(r[j]);
   __syncwarp();
   const int c = 4 * (lane & 7);
   const int col = col0 + c;
-  float bias[4], gv[4], gt[4];
+  // RoPE: the (cos, sin) of this lane's two pairs on its eight rows, all
+  // loaded through the read-only path before any output is stored, so that
+  // the loads overlap instead of queueing behind the stores
+  float2 rcs[KIND == EPI_ROPE_QKV ? 8 : 1][2];
+  if constexpr (KIND == EPI_ROPE_QKV) {
+    const int j0 = (col & (e.head_dim - 1)) >> 1;
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    bias[k] = e.bias ? e.bias[col + k] : 0.f;
-    gv[k] = KIND == EPI_GATED_RES ? e.gate_v[col + k] : 0.f;
-    gt[k] = KIND == EPI_GATED_RES ? e.gate_t[col + k] : 0.f;
+    for (int p = 0; p < 8; ++p) {
+      const int64_t grow = row0 + 4 * p + (lane >> 3) + e.row_base;
+      rcs[p][0] = rcs[p][1] = make_float2(1.f, 0.f);
+      if (col < 2 * e.d && grow >= e.rope_first_video && row0 + 4 * p + (lane >> 3) < g.M) {
+        const RopePos pp = rope_pos(e.rope, (int)(grow - e.rope_first_video));
+#pragma unroll
+        for (int q = 0; q < 2; ++q) rcs[p][q] = __ldg(&rope_cs_ptr(e.rope, pp, j0 + q));
+      }
+    }
   }
 #pragma unroll
   for (int p = 0; p < 8; ++p) {
@@ -212,36 +251,32 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
     const int64_t grow = row + e.row_base;
     float v[4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) v[k] = stage[rr * 33 + c + k] + bias[k];
+    for (int k = 0; k < 4; ++k) v[k] = stage[rr * 33 + c + k] + rc.bias[k];
     switch (KIND) {
       case EPI_GELU:
 #pragma unroll
         for (int k = 0; k < 4; ++k) v[k] = gelu_tanh<true>(v[k]);
         break;
       case EPI_ROPE_QKV:
-        if (col < 2 * e.d && grow >= e.rope_first_video) {
-          // one position decomposition per row; the four columns lie in one
-          // head (head_dim is a power of two, checked on the host)
-          const RopePos pp = rope_pos(e.rope, (int)(grow - e.rope_first_video));
-          const int j0 = (col & (e.head_dim - 1)) >> 1;
+        // (cos, sin) = (1, 0) on rows and columns that are not rotated; the
+        // four columns lie in one head (head_dim is a power of two)
 #pragma unroll
-          for (int k = 0; k < 4; k += 2) {
-            const float2 cs = rope_cs(e.rope, pp, j0 + (k >> 1));
-            const float x0 = v[k], x1 = v[k + 1];
-            v[k] = x0 * cs.x - x1 * cs.y;
-            v[k + 1] = x0 * cs.y + x1 * cs.x;
-          }
+        for (int k = 0; k < 4; k += 2) {
+          const float2 cs = rcs[p][k >> 1];
+          const float x0 = v[k], x1 = v[k + 1];
+          v[k] = x0 * cs.x - x1 * cs.y;
+          v[k + 1] = x0 * cs.y + x1 * cs.x;
         }
         break;
       case EPI_GATED_RES: {
         const bool text = grow < e.gate_split;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) v[k] = fmaf(text ? gt[k] : gv[k], v[k], rc.v[p][k]);
+        for (int k = 0; k < 4; ++k) v[k] = fmaf(text ? rc.gt[k] : rc.gv[k], v[k], res_value(rc, p, k));
         break;
       }
       case EPI_RES:
 #pragma unroll
-        for (int k = 0; k < 4; ++k) v[k] += rc.v[p][k];
+        for (int k = 0; k < 4; ++k) v[k] += res_value(rc, p, k);
         break;
       default:
         break;
@@ -255,7 +290,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
   __syncwarp();
 }
 
-template <int BN, int KIND>
+template <int BN, int KIND, bool R32>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
                    EpiDev e) {
@@ -347,23 +382,22 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const bool ok = mbar_wait(&acc_full[b], use & 1);
       tc_fence_after();
       const int64_t row0 = (int64_t)m_tile * BM + q * 32;
-      constexpr bool res = KIND == EPI_GATED_RES || KIND == EPI_RES;
       // this warp's chunks: columns [half * BN/2, (half + 1) * BN/2) of the tile, 32 at a time;
-      // residual values of chunk i+1 are loaded while chunk i is processed
+      // the global inputs of chunk i+1 (residual, bias, gates) are loaded while chunk i is processed
       constexpr int NC = BN / 64;
       const int cbeg = half * (BN / 2);
       const int lcol = 4 * (lane & 7);
-      auto process = [&](int i, const ResChunk& cur, ResChunk& nxt) {
+      auto process = [&](int i, const ResChunk<R32>& cur, ResChunk<R32>& nxt) {
         const int c = cbeg + 32 * i;
         uint32_t r[32];
         tmem_ld32(tmem + lane_base + b * BN + c, r);
         tmem_wait_ld();
         const int col0 = n_tile * BN + c;
-        if (res && i + 1 < NC && row0 < g.M && col0 + 32 < g.N) load_res_chunk(g, e, row0, col0 + 32 + lcol, nxt);
-        if (ok && row0 < g.M && col0 < g.N) epilogue_chunk<KIND>(g, e, stage, row0, col0, r, cur);
+        if (i + 1 < NC && row0 < g.M && col0 + 32 < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, col0 + 32 + lcol, nxt);
+        if (ok && row0 < g.M && col0 < g.N) epilogue_chunk<KIND, R32>(g, e, stage, row0, col0, r, cur);
       };
-      ResChunk rc0, rc1;
-      if (res && row0 < g.M && n_tile * BN + cbeg < g.N) load_res_chunk(g, e, row0, n_tile * BN + cbeg + lcol, rc0);
+      ResChunk<R32> rc0, rc1;
+      if (row0 < g.M && n_tile * BN + cbeg < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, n_tile * BN + cbeg + lcol, rc0);
 #pragma unroll 1
       for (int i = 0; i < NC; i += 2) {
         process(i, rc0, rc1);
@@ -431,16 +465,16 @@ int num_sms() {
   return n;
 }
 
-template <int BN, int KIND>
+template <int BN, int KIND, bool R32 = false>
 acid_status launch_tc_kind(const CUtensorMap& ta, const CUtensorMap& tb, const GemmDims& g, const Epilogue& epi,
                            int grid, cudaStream_t s) {
   using C = TcCfg<BN>;
   static bool attr_done = false;
   if (!attr_done) {
-    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN, KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN, KIND, R32>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
     attr_done = true;
   }
-  gemm_tc_kernel<BN, KIND><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
+  gemm_tc_kernel<BN, KIND, R32><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }
@@ -458,8 +492,12 @@ acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* 
   switch (epi.kind) {
     case EPI_GELU: return launch_tc_kind<BN, EPI_GELU>(ta, tb, g, epi, grid, s);
     case EPI_ROPE_QKV: return launch_tc_kind<BN, EPI_ROPE_QKV>(ta, tb, g, epi, grid, s);
-    case EPI_GATED_RES: return launch_tc_kind<BN, EPI_GATED_RES>(ta, tb, g, epi, grid, s);
-    case EPI_RES: return launch_tc_kind<BN, EPI_RES>(ta, tb, g, epi, grid, s);
+    case EPI_GATED_RES:
+      return epi.res_fp32 ? launch_tc_kind<BN, EPI_GATED_RES, true>(ta, tb, g, epi, grid, s)
+                          : launch_tc_kind<BN, EPI_GATED_RES, false>(ta, tb, g, epi, grid, s);
+    case EPI_RES:
+      return epi.res_fp32 ? launch_tc_kind<BN, EPI_RES, true>(ta, tb, g, epi, grid, s)
+                          : launch_tc_kind<BN, EPI_RES, false>(ta, tb, g, epi, grid, s);
     default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, g, epi, grid, s);
   }
 }

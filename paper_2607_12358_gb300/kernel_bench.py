@@ -4,8 +4,11 @@ warm-up), for tuning and for profiler captures of a single launch.
     python -m paper_2607_12358_gb300.kernel_bench attention --n 32760 --heads 12 --head-dim 128
     python -m paper_2607_12358_gb300.kernel_bench linear --m 32760 --k 1536 --n 8960 --epi gelu
     python -m paper_2607_12358_gb300.kernel_bench drift --rows 118800 --cols 3072 [--apply]
+    python -m paper_2607_12358_gb300.kernel_bench block --workload wan [--block-type wan]
 
-Inputs are random bf16 tensors created on the device.  Prints one JSON line.
+Inputs are random bf16 tensors created on the device (block: the synthetic
+full-size weights of one block of the named workload, a N(0,1) input and a
+N(0,1) stand-in time embedding).  Prints one JSON line.
 """
 
 from __future__ import annotations
@@ -37,7 +40,9 @@ def _time(fn, warmup, iters):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attention", "linear", "drift"])
+    ap.add_argument("kernel", choices=["attention", "linear", "drift", "block"])
+    ap.add_argument("--workload", default="wan", help="block: wan | cog | hv")
+    ap.add_argument("--block-type", default=None, help="block: wan | cog | hv_dual | hv_single")
     ap.add_argument("--n", type=int, default=32760)
     ap.add_argument("--nk", type=int, default=0, help="keys (attention); default = --n")
     ap.add_argument("--heads", type=int, default=12)
@@ -81,6 +86,25 @@ def main():
                    a.warmup, a.iters)
         flop = 2.0 * a.m * a.n * a.k
         out.update(shape=[a.m, a.k, a.n], epi=a.epi, ms=ms, tflops=flop / ms / 1e9)
+    elif a.kernel == "block":
+        import acid_synth as S
+
+        cfg = S.get_config(a.workload)
+        bt = a.block_type or {"wan": "wan", "cog": "cog", "hv": "hv_dual"}[a.workload]
+        w = S.block_weights(cfg, 0, seed=0, block_type=bt)
+        rows = cfg.n_video + (0 if bt == "wan" else cfg.n_text)
+        desc = acid.block_desc(cfg, bt)
+        blk = acid.DeviceBlock.upload(w, bt, torch.bfloat16, dev)
+        temb = torch.from_numpy(S.temb_vector(cfg, 0)).to(dev)
+        x0 = torch.randn(rows, cfg.d, device=dev, generator=gen).to(torch.bfloat16)
+        x = x0.clone()
+        ctx = None
+        if bt == "wan" and cfg.n_text:
+            ctx = torch.randn(cfg.n_text, cfg.d, device=dev, generator=gen).to(torch.bfloat16)
+        ws = torch.empty(acid.block_workspace_size(desc) + 1024, dtype=torch.uint8, device=dev)
+        ms = _time(lambda: acid.acid_dit_block_forward(desc, x.copy_(x0), temb, blk, ctx=ctx, workspace=ws),
+                   a.warmup, a.iters)
+        out.update(workload=a.workload, block_type=bt, rows=rows, ms=ms)
     else:
         n = a.rows * a.cols
         p = torch.randn(n, device=dev, generator=gen).to(torch.bfloat16)
