@@ -38,11 +38,12 @@ WORKLOAD = ("Wan-2.1-1.3B-shaped 480p step: 30 blocks, d=1536, 12 heads x 128, F
 CPU_SAMPLE_ROWS = 4096
 REF_SAMPLE_ROWS = 2048
 
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one ncu capture of a
-# self- and a cross-attention launch at this shape) per attention launch of
-# the step's 1:1 self/cross mix.  Valid only for the kernel source it was
-# measured on; any other source reports null.
-ATTN_TRAFFIC = {"source_sha256_16": "e1e6d248900fd9eb", "bytes_per_launch": (404.46e6 + 156.83e6) / 2}
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one ncu capture of
+# a self- and a cross-attention call at this shape, each call = the main
+# launch, the split tail launch and the merge) per attention call of the step's
+# 1:1 self/cross mix.  Valid only for the kernel source it was measured on; any
+# other source reports null.
+ATTN_TRAFFIC = {"source_sha256_16": "7f3819367c898c87", "bytes_per_launch": (438.40e6 + 165.79e6) / 2}
 
 
 def _attn_traffic():

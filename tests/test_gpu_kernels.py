@@ -76,6 +76,33 @@ def test_linear_bf16_epilogues(acid, epi):
     assert _rel_l2(got, ref) <= 4e-3
 
 
+@pytest.mark.parametrize("M,K,N", [(891, 320, 512), (1000, 64, 768), (2500, 1096, 1024)])
+@pytest.mark.parametrize("epi,fp32", [("bias", True), ("gelu", False), ("gated_res", False), ("gated_res", True),
+                                      ("res", True)])
+def test_linear_bf16_many_row_blocks(acid, M, K, N, epi, fp32):
+    """The 256-wide tile path over several row blocks, including an odd count
+    and a ragged last block (891 rows), fewer k-blocks than pipeline stages, a
+    K that wraps the stage ring several times with a partial last k-block
+    (1096), and every epilogue with bf16 and fp32 output/residual."""
+    rng = np.random.default_rng(M + 7 * K + N)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.1 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    g = rng.normal(size=N).astype(np.float32)
+    r = rng.normal(size=(M, N)).astype(np.float32)
+    if not fp32:
+        r = S.round_to_bf16(r)
+    has_res = epi in ("gated_res", "res")
+    res = (_f32(r) if fp32 else _bf(r)) if has_res else None
+    out = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), epilogue=epi, gate=_f32(g), residual=res, out=res,
+                                   out_fp32=fp32)
+    acc = O.linear(a, w, b)
+    ref = {"bias": acc, "gelu": O.gelu_tanh(acc), "gated_res": r + g * acc, "res": r + acc}[epi]
+    got = out.float().cpu().numpy()
+    tol = 1e-4 if (fp32 and epi != "gelu") else 2 ** -8
+    assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
+
+
 @pytest.mark.parametrize("M,K,N", [(1, 64, 64), (7, 8, 32), (127, 72, 96), (129, 200, 256), (3, 4104, 128)])
 def test_linear_bf16_edge_shapes(acid, M, K, N):
     """Single rows, K below / not a multiple of the 64-wide k-block (zero-filled
