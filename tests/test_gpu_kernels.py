@@ -148,7 +148,8 @@ def _attn_case(nq, nk, H, D, seed, qscale=1.0):
 
 @pytest.mark.parametrize("nq,nk,H,D,qscale", [(128, 128, 1, 128, 1.0), (300, 300, 2, 128, 1.0),
                                               (300, 257, 2, 64, 2.0), (1000, 512, 3, 128, 3.0),
-                                              (129, 1000, 2, 64, 4.0), (2048, 2048, 2, 128, 1.0)])
+                                              (129, 1000, 2, 64, 4.0), (2048, 2048, 2, 128, 1.0),
+                                              (1000, 2000, 3, 64, 3.0)])
 def test_attention_bf16(acid, nq, nk, H, D, qscale):
     q, k, v, ref = _attn_case(nq, nk, H, D, nq + nk, qscale)
     out = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), H)
