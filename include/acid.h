@@ -420,6 +420,17 @@ acid_status acid_denoise_loop_guided(const acid_model* m, const acid_loop_cfg* c
                                      acid_step_log* log_cond, acid_step_log* log_uncond,
                                      void* workspace, size_t workspace_bytes, acid_stream_t stream);
 
+/* The same guided generation as acid_denoise_loop_guided, launched as one
+ * CUDA graph (as acid_denoise_loop_graph): per step, both branches' signals
+ * and Algorithm 1 decisions are taken on the device, each selecting its own
+ * compute or reuse body.  Arithmetic and decisions are those of the
+ * host-driven guided loop; log entries have ms = NaN.  n_steps <= 1024. */
+acid_status acid_denoise_loop_guided_graph(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                                           const acid_loop_cfg* cfg_uncond, double guidance_scale,
+                                           void* latent, const void* text_cond, const void* text_uncond,
+                                           acid_step_log* log_cond, acid_step_log* log_uncond,
+                                           void* workspace, size_t workspace_bytes, acid_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

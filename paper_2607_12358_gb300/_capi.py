@@ -113,6 +113,10 @@ _PROTOS = {
     "acid_denoise_loop_guided": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg), C.POINTER(acid_loop_cfg),
                                            C.c_double, _P, _P, _P, C.POINTER(acid_step_log),
                                            C.POINTER(acid_step_log), _P, C.c_size_t, _P]),
+    "acid_denoise_loop_guided_graph": (C.c_int, [C.POINTER(acid_model), C.POINTER(acid_loop_cfg),
+                                                 C.POINTER(acid_loop_cfg), C.c_double, _P, _P, _P,
+                                                 C.POINTER(acid_step_log), C.POINTER(acid_step_log), _P, C.c_size_t,
+                                                 _P]),
 }
 
 _lib = None

@@ -413,15 +413,17 @@ class GuidedLoop:
 
 def acid_denoise_loop_guided(model: DeviceModel, cfg_cond, cfg_uncond, scale: float, latent: torch.Tensor,
                              text_cond: torch.Tensor | None = None, text_uncond: torch.Tensor | None = None,
-                             log: bool = True, stream=None) -> tuple[list[dict], list[dict]]:
-    """Runs a guided generation in place on latent; returns the two branches' step logs."""
+                             log: bool = True, stream=None, graph: bool = False) -> tuple[list[dict], list[dict]]:
+    """Runs a guided generation in place on latent; returns the two branches' step logs.
+    ``graph=True`` calls acid_denoise_loop_guided_graph (one CUDA graph, decisions on the device)."""
     _need_cuda(latent, text_cond, text_uncond)
     if latent.dtype != torch.float32:
         raise TypeError("latent must be fp32")
     n = cfg_cond.n_steps
     lc, lu = (A.acid_step_log * n)(), (A.acid_step_log * n)()
     ws, ptr, nbytes = _aligned_ws(guided_workspace_size(model), latent.device)
-    check(load().acid_denoise_loop_guided(C.byref(model.struct), C.byref(cfg_cond), C.byref(cfg_uncond), float(scale),
-                                          latent.data_ptr(), _ptr(text_cond), _ptr(text_uncond),
-                                          lc if log else None, lu if log else None, ptr, nbytes, _stream(stream)))
+    fn = load().acid_denoise_loop_guided_graph if graph else load().acid_denoise_loop_guided
+    check(fn(C.byref(model.struct), C.byref(cfg_cond), C.byref(cfg_uncond), float(scale), latent.data_ptr(),
+             _ptr(text_cond), _ptr(text_uncond), lc if log else None, lu if log else None, ptr, nbytes,
+             _stream(stream)))
     return ([log_to_dict(x) for x in lc], [log_to_dict(x) for x in lu]) if log else ([], [])

@@ -475,6 +475,18 @@ __global__ void guided_euler_kernel(float* lat, const float* __restrict__ vc, co
   }
 }
 
+// The same with dsigma read from device memory (graph-launched loops).
+__global__ void guided_euler_sig_kernel(float* lat, const float* __restrict__ vc, const float* __restrict__ vu,
+                                        int64_t n, float g, const double* sig, const int* step) {
+  const int i0 = *step;
+  const float dsig = (float)(sig[i0 + 1] - sig[i0]);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const float u = vu[i];
+    lat[i] = fmaf(dsig, fmaf(g, vc[i] - u, u), lat[i]);
+  }
+}
+
 // dsigma = sigma[step + 1] - sigma[step] with the step index read from device memory
 __global__ void euler_sig_kernel(float* lat, const float* __restrict__ v, int64_t n, const double* sig,
                                  const int* step) {
@@ -684,6 +696,13 @@ acid_status euler_update(float* latent, const float* v, int64_t n, float dsigma,
 acid_status guided_euler_update(float* latent, const float* v_cond, const float* v_uncond, int64_t n, float scale,
                                float dsigma, cudaStream_t s) {
   guided_euler_kernel<<<grid_for(n), kThreads, 0, s>>>(latent, v_cond, v_uncond, n, scale, dsigma);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status guided_euler_update_sig(float* latent, const float* v_cond, const float* v_uncond, int64_t n, float scale,
+                                   const double* sig, const int* step, cudaStream_t s) {
+  guided_euler_sig_kernel<<<grid_for(n), kThreads, 0, s>>>(latent, v_cond, v_uncond, n, scale, sig, step);
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }

@@ -118,6 +118,8 @@ acid_status unpatchify_euler(const float* vtok, float* v_out, float* latent, int
 acid_status euler_update(float* latent, const float* v, int64_t n, float dsigma, cudaStream_t s);
 acid_status guided_euler_update(float* latent, const float* v_cond, const float* v_uncond, int64_t n, float scale,
                                float dsigma, cudaStream_t s);
+acid_status guided_euler_update_sig(float* latent, const float* v_cond, const float* v_uncond, int64_t n, float scale,
+                                   const double* sig, const int* step, cudaStream_t s);
 // Variants that read the step index from device memory (graph-launched loops):
 // t = 1000 sig[*step]; dsigma = sig[*step + 1] - sig[*step].
 acid_status euler_update_sig(float* latent, const float* v, int64_t n, const double* sig, const int* step,

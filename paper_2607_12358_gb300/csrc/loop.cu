@@ -776,8 +776,11 @@ __global__ void easycache_rate_kernel(DevLoop* st, const double* dres) {
   st->have_rate = 1;
 }
 
-__global__ void advance_kernel(DevLoop* st, cudaGraphConditionalHandle h_loop) {
+// Next step: the step index of the branch (and of the second branch of a
+// guided generation), and the WHILE condition.
+__global__ void advance_kernel(DevLoop* st, DevLoop* st2, cudaGraphConditionalHandle h_loop) {
   st->step += 1;
+  if (st2) st2->step += 1;
   cudaGraphSetConditional(h_loop, st->step < st->n_steps ? 1u : 0u);
 }
 
@@ -809,9 +812,13 @@ struct GraphCapture {
   }
 };
 
-// Records one step into `body` (captured on gc.main; conditional bodies on gc.side).
-acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& w, float* latent, GraphCapture& gc,
-                         cudaGraph_t body, cudaGraphConditionalHandle h_loop) {
+// Records, into the graph `body` that gc.main is capturing, one branch's part
+// of a step: its inputs, signal and Algorithm 1 decision, the compute or reuse
+// body of an IF/ELSE node (captured on gc.side), and its velocity in w.v[0]
+// together with the copies that keep the previous step's values.  The Euler
+// update is left to the caller.
+acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& w, float* latent,
+                           GraphCapture& gc, cudaGraph_t body) {
   const Shape sh = shape_of(m);
   const int dt = m.block.dtype;
   cudaStream_t s = gc.main, s2 = gc.side;
@@ -821,7 +828,6 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
   cudaGraphConditionalHandle h_compute;
   ACID_CUDA(cudaGraphConditionalHandleCreate(&h_compute, body, 0, 0));
 
-  ACID_CUDA(cudaStreamBeginCaptureToGraph(s, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
   // ---- step inputs: temb, patch embedding
   ACID_TRY(timestep_sinusoid_sig(w.sinus, w.sig, step, m.time_freq_dim, s));
   ACID_TRY(gemv(dt, m.time1.w, m.time1.b, w.sinus, w.temb_h, sh.d, m.time_freq_dim, false, s));
@@ -897,7 +903,7 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
     ACID_TRY(add_mixed(ACID_FP32, latent, ACID_FP32, w.offset, ACID_FP32, v, sh.latent, 1.0f, s2));
   ACID_CUDA(cudaStreamEndCapture(s2, &tmp));
 
-  // ---- output: velocity and the Euler update, then the next step
+  // ---- output: the velocity, and the previous step's values
   if (cfg.method == ACID_METHOD_TEACACHE) {
     ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s));
   } else if (cfg.method == ACID_METHOD_DICACHE) {
@@ -907,55 +913,71 @@ acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& 
     ACID_CUDA(cudaMemcpyAsync(w.x_prev, latent, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
     ACID_CUDA(cudaMemcpyAsync(v_prev, v, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
   }
-  ACID_TRY(euler_update_sig(latent, v, sh.latent, w.sig, step, s));
-  advance_kernel<<<1, 1, 0, s>>>(w.dev, h_loop);
+  return ACID_OK;
+}
+
+// One sampler step into `body`: the branch, the Euler update, the next step.
+acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& w, float* latent, GraphCapture& gc,
+                         cudaGraph_t body, cudaGraphConditionalHandle h_loop) {
+  cudaStream_t s = gc.main;
+  ACID_CUDA(cudaStreamBeginCaptureToGraph(s, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  ACID_TRY(capture_branch(m, cfg, w, latent, gc, body));
+  ACID_TRY(euler_update_sig(latent, w.v[0], shape_of(m).latent, w.sig, &w.dev->step, s));
+  advance_kernel<<<1, 1, 0, s>>>(w.dev, nullptr, h_loop);
   ACID_CHECK_LAUNCH();
+  cudaGraph_t tmp;
   ACID_CUDA(cudaStreamEndCapture(s, &tmp));
   return ACID_OK;
 }
 
-}  // namespace
-}  // namespace acid
+// One guided step: both branches on x_i, then x_{i+1} = x_i + dsigma (v_u + g (v_c - v_u)).
+acid_status capture_guided_step(const acid_model& m, const acid_loop_cfg& cc, const acid_loop_cfg& cu, float scale,
+                                LoopWs& wc, LoopWs& wu, float* latent, GraphCapture& gc, cudaGraph_t body,
+                                cudaGraphConditionalHandle h_loop) {
+  cudaStream_t s = gc.main;
+  ACID_CUDA(cudaStreamBeginCaptureToGraph(s, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+  ACID_TRY(capture_branch(m, cc, wc, latent, gc, body));
+  ACID_TRY(capture_branch(m, cu, wu, latent, gc, body));
+  ACID_TRY(guided_euler_update_sig(latent, wc.v[0], wu.v[0], shape_of(m).latent, scale, wc.sig, &wc.dev->step, s));
+  advance_kernel<<<1, 1, 0, s>>>(wc.dev, wu.dev, h_loop);
+  ACID_CHECK_LAUNCH();
+  cudaGraph_t tmp;
+  ACID_CUDA(cudaStreamEndCapture(s, &tmp));
+  return ACID_OK;
+}
 
-extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_loop_cfg* cfg, void* latent_v,
-                                               const void* text, acid_step_log* log, void* workspace,
-                                               size_t workspace_bytes, acid_stream_t stream) {
-  clear_error();
-  ACID_REQUIRE(m && cfg && latent_v, ACID_ERR_INVALID_ARG, "acid_denoise_loop_graph: null argument");
-  ACID_TRY(validate_cfg(*cfg));
-  ACID_REQUIRE(cfg->n_steps <= kMaxGraphSteps, ACID_ERR_UNSUPPORTED,
-               "acid_denoise_loop_graph: at most " + std::to_string(kMaxGraphSteps) + " steps");
-  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_denoise_loop_graph: latent must be 16-byte aligned");
-  acid_loop_state st;
-  ACID_TRY(acid_loop_begin(m, cfg, text, &st, workspace, workspace_bytes, stream));
-  LoopWs w = loop_layout(*m, workspace);
-  cudaStream_t s = (cudaStream_t)stream;
-  const Shape sh = shape_of(*m);
-  // device state, noise levels and forced decisions
+// Device-side loop state, noise levels, forced decisions and threshold
+// schedule of one branch; `stream` is synchronised (host sources are stack memory).
+acid_status setup_graph_state(const acid_model& m, const acid_loop_cfg& cfg, const LoopWs& w, cudaStream_t s) {
+  const Shape sh = shape_of(m);
   DevLoop d = {};
-  d.n_steps = cfg->n_steps;
-  d.warmup = cfg->warmup;
-  d.method = cfg->method;
-  d.force_last = cfg->force_last;
-  d.use_forced = cfg->forced != nullptr;
-  d.use_tau_sched = cfg->tau_schedule != nullptr;
-  d.tau_low = cfg->tau_low;
-  d.tau_high = cfg->tau_high;
-  d.delta = cfg->delta;
+  d.n_steps = cfg.n_steps;
+  d.warmup = cfg.warmup;
+  d.method = cfg.method;
+  d.force_last = cfg.force_last;
+  d.use_forced = cfg.forced != nullptr;
+  d.use_tau_sched = cfg.tau_schedule != nullptr;
+  d.tau_low = cfg.tau_low;
+  d.tau_high = cfg.tau_high;
+  d.delta = cfg.delta;
   d.latent_n = (double)sh.latent;
-  d.poly_n = cfg->signal_poly_n;
-  for (int j = 0; j < cfg->signal_poly_n; ++j) d.poly[j] = cfg->signal_poly[j];
+  d.poly_n = cfg.signal_poly_n;
+  for (int j = 0; j < cfg.signal_poly_n; ++j) d.poly[j] = cfg.signal_poly[j];
   double sig[kMaxGraphSteps + 1];
-  for (int i = 0; i <= cfg->n_steps; ++i) sig[i] = sigma_at(*cfg, i);
+  for (int i = 0; i <= cfg.n_steps; ++i) sig[i] = sigma_at(cfg, i);
   ACID_CUDA(cudaMemcpyAsync(w.dev, &d, sizeof(d), cudaMemcpyHostToDevice, s));
-  ACID_CUDA(cudaMemcpyAsync(w.sig, sig, sizeof(double) * (cfg->n_steps + 1), cudaMemcpyHostToDevice, s));
-  if (cfg->forced)
-    ACID_CUDA(cudaMemcpyAsync(w.forced, cfg->forced, cfg->n_steps, cudaMemcpyHostToDevice, s));
-  if (cfg->tau_schedule)
-    ACID_CUDA(cudaMemcpyAsync(w.tau_sched, cfg->tau_schedule, sizeof(double) * cfg->n_steps,
-                              cudaMemcpyHostToDevice, s));
-  ACID_CUDA(cudaStreamSynchronize(s));  // host sources above are stack memory
+  ACID_CUDA(cudaMemcpyAsync(w.sig, sig, sizeof(double) * (cfg.n_steps + 1), cudaMemcpyHostToDevice, s));
+  if (cfg.forced) ACID_CUDA(cudaMemcpyAsync(w.forced, cfg.forced, cfg.n_steps, cudaMemcpyHostToDevice, s));
+  if (cfg.tau_schedule)
+    ACID_CUDA(cudaMemcpyAsync(w.tau_sched, cfg.tau_schedule, sizeof(double) * cfg.n_steps, cudaMemcpyHostToDevice, s));
+  ACID_CUDA(cudaStreamSynchronize(s));
+  return ACID_OK;
+}
 
+// Builds the WHILE graph around `record` (which captures one step into the
+// body), launches it on `stream`, synchronises and destroys it.
+template <typename Record>
+acid_status run_graph(cudaStream_t stream, Record record) {
   GraphCapture gc;
   ACID_CUDA(cudaStreamCreateWithFlags(&gc.main, cudaStreamNonBlocking));
   ACID_CUDA(cudaStreamCreateWithFlags(&gc.side, cudaStreamNonBlocking));
@@ -981,7 +1003,7 @@ extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_l
       set_error("cudaGraphAddNode (while) failed");
       break;
     }
-    rc = capture_step(*m, *cfg, w, static_cast<float*>(latent_v), gc, p.conditional.phGraph_out[0], h_loop);
+    rc = record(gc, p.conditional.phGraph_out[0], h_loop);
     if (rc != ACID_OK) {
       cudaGraph_t junk;
       cudaStreamEndCapture(gc.side, &junk);
@@ -994,10 +1016,8 @@ extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_l
       set_error(std::string("cudaGraphInstantiate: ") + cudaGetErrorString(e));
       break;
     }
-    e = cudaGraphLaunch(exec, s);
-    if (e == cudaSuccess && log)
-      e = cudaMemcpyAsync(log, w.dlog, sizeof(acid_step_log) * cfg->n_steps, cudaMemcpyDeviceToHost, s);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    e = cudaGraphLaunch(exec, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
     if (e != cudaSuccess) {
       rc = ACID_ERR_CUDA;
       set_error(std::string("graph launch: ") + cudaGetErrorString(e));
@@ -1006,4 +1026,65 @@ extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_l
   if (exec) cudaGraphExecDestroy(exec);
   if (g) cudaGraphDestroy(g);
   return rc;
+}
+
+}  // namespace
+}  // namespace acid
+
+extern "C" acid_status acid_denoise_loop_graph(const acid_model* m, const acid_loop_cfg* cfg, void* latent_v,
+                                               const void* text, acid_step_log* log, void* workspace,
+                                               size_t workspace_bytes, acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m && cfg && latent_v, ACID_ERR_INVALID_ARG, "acid_denoise_loop_graph: null argument");
+  ACID_TRY(validate_cfg(*cfg));
+  ACID_REQUIRE(cfg->n_steps <= kMaxGraphSteps, ACID_ERR_UNSUPPORTED,
+               "acid_denoise_loop_graph: at most " + std::to_string(kMaxGraphSteps) + " steps");
+  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED, "acid_denoise_loop_graph: latent must be 16-byte aligned");
+  acid_loop_state st;
+  ACID_TRY(acid_loop_begin(m, cfg, text, &st, workspace, workspace_bytes, stream));
+  LoopWs w = loop_layout(*m, workspace);
+  cudaStream_t s = (cudaStream_t)stream;
+  ACID_TRY(setup_graph_state(*m, *cfg, w, s));
+  float* latent = static_cast<float*>(latent_v);
+  ACID_TRY(run_graph(s, [&](GraphCapture& gc, cudaGraph_t body, cudaGraphConditionalHandle h_loop) {
+    return capture_step(*m, *cfg, w, latent, gc, body, h_loop);
+  }));
+  if (log) {
+    ACID_CUDA(cudaMemcpyAsync(log, w.dlog, sizeof(acid_step_log) * cfg->n_steps, cudaMemcpyDeviceToHost, s));
+    ACID_CUDA(cudaStreamSynchronize(s));
+  }
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_denoise_loop_guided_graph(const acid_model* m, const acid_loop_cfg* cfg_cond,
+                                                      const acid_loop_cfg* cfg_uncond, double guidance_scale,
+                                                      void* latent_v, const void* text_cond, const void* text_uncond,
+                                                      acid_step_log* log_cond, acid_step_log* log_uncond,
+                                                      void* workspace, size_t workspace_bytes, acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(m && cfg_cond && cfg_uncond && latent_v, ACID_ERR_INVALID_ARG,
+               "acid_denoise_loop_guided_graph: null argument");
+  ACID_REQUIRE(cfg_cond->n_steps <= kMaxGraphSteps, ACID_ERR_UNSUPPORTED,
+               "acid_denoise_loop_guided_graph: at most " + std::to_string(kMaxGraphSteps) + " steps");
+  ACID_REQUIRE(aligned(latent_v, 16), ACID_ERR_UNSUPPORTED,
+               "acid_denoise_loop_guided_graph: latent must be 16-byte aligned");
+  ACID_REQUIRE(std::isfinite(guidance_scale), ACID_ERR_INVALID_ARG,
+               "acid_denoise_loop_guided_graph: guidance scale not finite");
+  acid_loop_state sc, su;
+  ACID_TRY(acid_guided_begin(m, cfg_cond, cfg_uncond, text_cond, text_uncond, &sc, &su, workspace, workspace_bytes,
+                             stream));
+  LoopWs wc, wu;
+  ACID_TRY(guided_check(m, cfg_cond, cfg_uncond, workspace, workspace_bytes, &wc, &wu));
+  cudaStream_t s = (cudaStream_t)stream;
+  ACID_TRY(setup_graph_state(*m, *cfg_cond, wc, s));
+  ACID_TRY(setup_graph_state(*m, *cfg_uncond, wu, s));
+  float* latent = static_cast<float*>(latent_v);
+  ACID_TRY(run_graph(s, [&](GraphCapture& gc, cudaGraph_t body, cudaGraphConditionalHandle h_loop) {
+    return capture_guided_step(*m, *cfg_cond, *cfg_uncond, (float)guidance_scale, wc, wu, latent, gc, body, h_loop);
+  }));
+  const int n = cfg_cond->n_steps;
+  if (log_cond) ACID_CUDA(cudaMemcpyAsync(log_cond, wc.dlog, sizeof(acid_step_log) * n, cudaMemcpyDeviceToHost, s));
+  if (log_uncond) ACID_CUDA(cudaMemcpyAsync(log_uncond, wu.dlog, sizeof(acid_step_log) * n, cudaMemcpyDeviceToHost, s));
+  ACID_CUDA(cudaStreamSynchronize(s));
+  return ACID_OK;
 }

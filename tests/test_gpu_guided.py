@@ -11,6 +11,8 @@ caches against the oracle's guided loop.
 * step-wise driving equals the whole-loop call.
 * bf16 small Wan shape: each branch's decisions are what the oracle
   controller takes on that branch's own logged signals.
+* acid_denoise_loop_guided_graph (one CUDA graph, both decisions on the
+  device) equals the host-driven guided loop bit for bit.
 """
 
 import numpy as np
@@ -150,3 +152,56 @@ def test_bf16_guided_replay(acid, method):
     if method == "teacache":
         assert [l["signal"] for l in lc][W:] == [l["signal"] for l in lu][W:]
     assert np.isfinite(got).all()
+
+
+def _same_logs(la, lb):
+    for x, y in zip(la, lb):
+        assert x["computed"] == y["computed"] and x["warmup"] == y["warmup"] and x["forced"] == y["forced"]
+        for k in ("signal", "dsignal", "tau", "sigma", "t"):
+            assert (x[k] != x[k] and y[k] != y[k]) or x[k] == y[k], (k, x, y)
+
+
+@pytest.mark.parametrize("method", ["teacache", "easycache", "dicache"])
+def test_toy_guided_graph_equals_host_loop(acid, method):
+    """The graph-launched guided generation (decisions on the device) runs the
+    same kernels in the same order as the host-driven one: identical logs and
+    a bit-identical latent."""
+    cfg = _toy(method, steps=10)
+    w = S.model_weights(cfg, 48)
+    lat, tc, tu = S.latent(cfg, 48), S.text(cfg, 48), S.text(cfg, 49)
+    model = acid.DeviceModel(cfg, w, DEV)
+    outs = []
+    for graph in (False, True):
+        cc, kc = acid.loop_cfg(cfg, method=method)
+        cu, ku = acid.loop_cfg(cfg, method=method, forced=[None] * 7 + [True] + [None] * 2)
+        x = torch.from_numpy(lat).to(DEV)
+        t_c = torch.from_numpy(tc).to(DEV)
+        t_u = torch.from_numpy(tu).to(DEV)
+        lc, lu = acid.acid_denoise_loop_guided(model, cc, cu, 3.5, x, t_c, t_u, graph=graph)
+        acid.check_device_error()
+        outs.append((x.cpu().numpy(), lc, lu))
+    (xa, lca, lua), (xb, lcb, lub) = outs
+    _same_logs(lca, lcb)
+    _same_logs(lua, lub)
+    np.testing.assert_array_equal(xa, xb)
+    assert lub[7]["forced"] and lub[7]["computed"]
+
+
+def test_bf16_guided_graph_equals_host_loop(acid):
+    over = dict(d=256, heads=2, ffn=512, latent_f=3, latent_h=16, latent_w=22, steps=8)
+    cfg = S.get_config("wan", n_blocks=2, n_text=40, d_text=256, **over)
+    w = S.model_weights(cfg, 50)
+    model = acid.DeviceModel(cfg, w, DEV)
+    t_c = torch.from_numpy(S.text(cfg, 50)).to(DEV, torch.bfloat16)
+    t_u = torch.from_numpy(S.text(cfg, 51)).to(DEV, torch.bfloat16)
+    outs = []
+    for graph in (False, True):
+        cc, kc = acid.loop_cfg(cfg)
+        cu, ku = acid.loop_cfg(cfg)
+        x = torch.from_numpy(S.latent(cfg, 50)).to(DEV)
+        lc, lu = acid.acid_denoise_loop_guided(model, cc, cu, 5.0, x, t_c, t_u, graph=graph)
+        acid.check_device_error()
+        outs.append((x.cpu().numpy(), lc, lu))
+    _same_logs(outs[0][1], outs[1][1])
+    _same_logs(outs[0][2], outs[1][2])
+    np.testing.assert_array_equal(outs[0][0], outs[1][0])
