@@ -307,6 +307,18 @@ def run_ours(args) -> None:
     acid_ms = e0.elapsed_time(e1)
     computed = sum(int(x.computed) for x in logs)
 
+    # ---- the same every-step-computed generation as one CUDA graph (signal and
+    # decision on the device); the wall time includes building and
+    # instantiating the graph
+    c4, keep4 = acid.loop_cfg(cfg, n_steps=K, tau_low=-1.0, tau_high=-1.0)
+    lat4 = torch.from_numpy(lat0).to(dev)
+    barrier()
+    t0 = time.perf_counter()
+    acid.acid_denoise_loop(model, c4, lat4, text, log=False, graph=True)
+    barrier()
+    graph_s = time.perf_counter() - t0
+    acid.check_device_error()
+
     if rank != 0:
         return
     peaks, src = _peaks()
@@ -333,6 +345,9 @@ def run_ours(args) -> None:
         "acid_mode": {"steps_per_s": K / (acid_ms / 1000.0), "computed_steps": computed, "of": K,
                       "tau_low": cfg.tau_low, "tau_high": cfg.tau_high, "delta": cfg.delta,
                       "note": "random weights: the skip rate says nothing about a trained model"},
+        "graph_mode": {"steps_per_s": world * K / graph_s,
+                       "note": "the same K steps, every step computed, as one CUDA graph (WHILE over steps, "
+                               "IF/ELSE per decision); wall time including graph build and instantiation"},
         "e2e": {"value": world * K / e2e_s, "unit": UNIT, "h2d_bytes_per_step": lat_bytes,
                 "d2h_bytes_per_step": lat_bytes},
         "gpu_launches": launches,
