@@ -5,8 +5,9 @@
  *
  * The library computes, on one GPU, the per-step evaluation of a video DiT
  * denoiser and the cheap drift reductions that decide whether a step is
- * computed or reused (Sec. 2 "TeaCache" / "EasyCache", Sec. 3.3,
- * Algorithm 1).  Every call takes plain pointers and sizes.
+ * computed or reused (Sec. 2 "TeaCache" / "EasyCache" / "DiCache", Sec. 3.3,
+ * Algorithm 1), around an Euler flow-matching sampler, with or without
+ * classifier-free guidance.  Every call takes plain pointers and sizes.
  *
  * Conventions shared by all entry points
  *  - Pointers named "device" must point to memory on the current CUDA device.
