@@ -36,7 +36,6 @@ namespace {
 
 constexpr int kTileQ = 128;  // query rows per tile (two tiles per CTA)
 constexpr int kBQ = 2 * kTileQ;
-constexpr int kBKV = 128;  // keys per K/V tile
 constexpr int kAttnThreads = 320;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kAttnPartCtas = kAttnSplitCtas;  // CTAs of a split tail wave (partials workspace capacity)
@@ -61,22 +60,32 @@ struct AttnDev {
 
 template <int D>
 struct AttnCfg {
-  static constexpr int CH = D / 64;                 // 64-column chunks per row
-  static constexpr int CHUNK_BYTES = 128 * 128;     // 128 rows x 128 bytes
-  static constexpr int T_BYTES = CH * CHUNK_BYTES;  // one 128-row tile of Q, K or V
-  static constexpr int OFF_Q = 0;                   // Q_a, Q_b
-  static constexpr int OFF_K = OFF_Q + 2 * T_BYTES;
-  static constexpr int OFF_V = OFF_K + 2 * T_BYTES;
-  static constexpr int OFF_BAR = OFF_V + 2 * T_BYTES;
+  // Keys per K/V tile.  Head dim 128: 128-key tiles, one CTA per SM (S and O
+  // of both query tiles fill TMEM).  Head dim 64: 64-key tiles, so a CTA needs
+  // 256 TMEM columns and about 64 KB of shared memory and two CTAs share an
+  // SM, four query tiles in flight: at this head dim the exponentials, not
+  // the MMAs, set the pace and need more warps to overlap.
+  static constexpr int BKV = D <= 64 ? 64 : 128;
+  static constexpr int CTAS_PER_SM = D <= 64 ? 2 : 1;
+  static constexpr int CH = D / 64;                  // 64-column chunks per row
+  static constexpr int CHUNK_Q = 128 * 128;          // 128 rows x 128 bytes
+  static constexpr int CHUNK_KV = BKV * 128;         // BKV rows x 128 bytes
+  static constexpr int T_BYTES = CH * CHUNK_Q;       // one 128-row tile of Q
+  static constexpr int KV_BYTES = CH * CHUNK_KV;     // one K or V tile
+  static constexpr int OFF_Q = 0;                    // Q_a, Q_b
+  static constexpr int OFF_K = OFF_Q + 2 * T_BYTES;  // 2-deep rings
+  static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_V + 2 * KV_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  // TMEM columns: S_a [0,128), S_b [128,256) (P_t over the first 64 columns of
-  // S_t), O_a [256, 256+D), O_b [384, 384+D)
-  static constexpr uint32_t TMEM_COLS = 512;
-  static constexpr uint32_t S_COL = 0, O_COL = 256;
+  // TMEM columns: S_a [0,BKV), S_b [BKV,2BKV) (P_t over the first BKV/2
+  // columns of S_t), O_a [2BKV, 2BKV+D), O_b [2BKV+D, 2BKV+2D)
+  static constexpr uint32_t S_COL = 0, O_COL = 2 * BKV;
+  static constexpr uint32_t TMEM_COLS = 2 * BKV + 2 * D;
+  __host__ __device__ static constexpr uint32_t o_col(int t) { return O_COL + t * D; }
 };
 
 template <int D>
-__global__ void __launch_bounds__(kAttnThreads, 1)
+__global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, AttnDev a) {
   using C = AttnCfg<D>;
@@ -99,7 +108,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int item = a.item_base + (int)blockIdx.x / a.splits, split = (int)blockIdx.x % a.splits;
   const int qt = item % a.nqp, h = item / a.nqp;
-  const int nkv_all = (int)((a.nk + kBKV - 1) / kBKV);
+  const int nkv_all = (int)((a.nk + C::BKV - 1) / C::BKV);
   const int jb = (int)((int64_t)split * nkv_all / a.splits);  // this CTA's key tiles [jb, jb + nkv)
   const int nkv = (int)((int64_t)(split + 1) * nkv_all / a.splits) - jb;
 
@@ -130,41 +139,42 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_expect_tx(q_full, 2 * C::T_BYTES);
       for (int t = 0; t < 2; ++t)
         for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sQ + t * C::T_BYTES + c * C::CHUNK_BYTES, &tmQ, q_full, a.q_col + h * D + c * 64,
+          tma_load_2d(sQ + t * C::T_BYTES + c * C::CHUNK_Q, &tmQ, q_full, a.q_col + h * D + c * 64,
                       qt * kBQ + t * kTileQ);
       for (int j = 0; j < nkv; ++j) {
         const int st = j & 1, round = j >> 1;
         if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) break;
-        mbar_expect_tx(&k_full[st], C::T_BYTES);
+        mbar_expect_tx(&k_full[st], C::KV_BYTES);
         for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sK + st * C::T_BYTES + c * C::CHUNK_BYTES, &tmK, &k_full[st], a.k_col + h * D + c * 64,
-                      (jb + j) * kBKV);
+          tma_load_2d(sK + st * C::KV_BYTES + c * C::CHUNK_KV, &tmK, &k_full[st], a.k_col + h * D + c * 64,
+                      (jb + j) * C::BKV);
         if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) break;
-        mbar_expect_tx(&v_full[st], C::T_BYTES);
+        mbar_expect_tx(&v_full[st], C::KV_BYTES);
         for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sV + st * C::T_BYTES + c * C::CHUNK_BYTES, &tmV, &v_full[st], a.v_col + h * D + c * 64,
-                      (jb + j) * kBKV);
+          tma_load_2d(sV + st * C::KV_BYTES + c * C::CHUNK_KV, &tmV, &v_full[st], a.v_col + h * D + c * 64,
+                      (jb + j) * C::BKV);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------------------------------- MMA issuer
-      constexpr uint32_t idesc_s = idesc_bf16_f32(128, kBKV, false, false);
+      constexpr uint32_t idesc_s = idesc_bf16_f32(128, C::BKV, false, false);
       constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
       // Shared-memory descriptors are built once; an operand at byte offset o
       // from a base is the base descriptor plus o >> 4 (the 14-bit address
       // field cannot overflow: shared memory ends below 256 KB).
       const uint64_t qdesc = smem_desc_sw128(smem_u32(sQ), 16, 1024);
       const uint64_t kdesc = smem_desc_sw128(smem_u32(sK), 16, 1024);
-      const uint64_t vdesc = smem_desc_sw128(smem_u32(sV), C::CHUNK_BYTES, 1024);
+      const uint64_t vdesc = smem_desc_sw128(smem_u32(sV), C::CHUNK_KV, 1024);
       // S_t(j) = Q_t K_j^T into the S region of tile t
       auto issue_s = [&](int t, int j) {
         const uint64_t a0 = qdesc + (uint64_t)((t * C::T_BYTES) >> 4);
-        const uint64_t b0 = kdesc + (uint64_t)(((j & 1) * C::T_BYTES) >> 4);
-        const uint32_t d = tmem + C::S_COL + t * kBKV;
+        const uint64_t b0 = kdesc + (uint64_t)(((j & 1) * C::KV_BYTES) >> 4);
+        const uint32_t d = tmem + C::S_COL + t * C::BKV;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t off = (uint64_t)(((kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32) >> 4);
-          mma_bf16_ss(d, a0 + off, b0 + off, idesc_s, kk != 0);
+          const uint64_t off_a = (uint64_t)(((kk >> 2) * C::CHUNK_Q + (kk & 3) * 32) >> 4);
+          const uint64_t off_b = (uint64_t)(((kk >> 2) * C::CHUNK_KV + (kk & 3) * 32) >> 4);
+          mma_bf16_ss(d, a0 + off_a, b0 + off_b, idesc_s, kk != 0);
         }
         mma_commit(&s_full[t]);
       };
@@ -182,10 +192,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           if (t == 0 && !mbar_wait(&v_full[st], (j >> 1) & 1)) { ok = false; break; }
           tc_fence_after();
           // O_t += P_t V_j: P_t (128 x 128 keys) from TMEM, V_j MN-major from shared memory
-          const uint64_t b0 = vdesc + (uint64_t)((st * C::T_BYTES) >> 4);
-          const uint32_t d = tmem + C::O_COL + t * 128, p0 = tmem + C::S_COL + t * kBKV;
+          const uint64_t b0 = vdesc + (uint64_t)((st * C::KV_BYTES) >> 4);
+          const uint32_t d = tmem + C::o_col(t), p0 = tmem + C::S_COL + t * C::BKV;
 #pragma unroll
-          for (int kk = 0; kk < kBKV / 16; ++kk)
+          for (int kk = 0; kk < C::BKV / 16; ++kk)
             mma_bf16_ts(d, p0 + kk * 8, b0 + (uint64_t)((kk * 16 * 128) >> 4), idesc_o, (j | kk) != 0);
           mma_commit(&pv_done[t]);
           if (t == 1) mma_commit(&v_empty[st]);
@@ -203,8 +213,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int q = warp & 3;
     const int r = q * 32 + lane;  // row within the query tile == TMEM lane
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-    const uint32_t s_addr = tmem + lane_base + C::S_COL + t * kBKV;
-    const uint32_t o_addr = tmem + lane_base + C::O_COL + t * 128;
+    const uint32_t s_addr = tmem + lane_base + C::S_COL + t * C::BKV;
+    const uint32_t o_addr = tmem + lane_base + C::o_col(t);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     // One key tile; the masked variant (keys past the end of the sequence)
@@ -215,16 +225,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       // after PV_t(j-1)) so that the final parity wait is never two phases ahead
       if (j > 0 && !mbar_wait(&pv_done[t], (j - 1) & 1)) return false;
       tc_fence_after();
-      float s[kBKV];
+      float s[C::BKV];
 #pragma unroll
-      for (int c = 0; c < kBKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
+      for (int c = 0; c < C::BKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
       tmem_wait_ld();
       bool resc = false;
       float f = 1.0f;
       if constexpr (decltype(masked)::value) {
-        const int valid = (int)(a.nk - (int64_t)(jb + j) * kBKV);  // keys of the last tile
+        const int valid = (int)(a.nk - (int64_t)(jb + j) * C::BKV);  // keys of the last tile
 #pragma unroll
-        for (int i = 0; i < kBKV; ++i)
+        for (int i = 0; i < C::BKV; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
       // e = s * scale - m_run in place (packed pairs; the first tile uses 0 as
@@ -239,7 +249,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint64_t nm2 = f2_pack(-mref, -mref);
         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int i = 0; i < kBKV / 2; ++i) {
+        for (int i = 0; i < C::BKV / 2; ++i) {
           f2_unpack(f2_fma(f2_pack(s[2 * i], s[2 * i + 1]), sc2, nm2), s[2 * i], s[2 * i + 1]);
           m4[i & 3] = fmax3(m4[i & 3], s[2 * i], s[2 * i + 1]);
         }
@@ -253,14 +263,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           m_run = mref + me;
           const uint64_t sh2 = f2_pack(-me, -me);
 #pragma unroll
-          for (int i = 0; i < kBKV / 2; ++i) f2_unpack(f2_add(f2_pack(s[2 * i], s[2 * i + 1]), sh2), s[2 * i], s[2 * i + 1]);
+          for (int i = 0; i < C::BKV / 2; ++i) f2_unpack(f2_add(f2_pack(s[2 * i], s[2 * i + 1]), sh2), s[2 * i], s[2 * i + 1]);
         }
       }
       // P = 2^e as bf16 pairs over the first 64 columns of S_t, with the row
       // sum as packed fp32 pairs
       uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
+      for (int half = 0; half < C::BKV / 64; ++half) {
         uint32_t pk[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
@@ -294,7 +304,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_arrive(&p_full[t]);
           return true;
     };
-    const bool partial_last = (int64_t)(jb + nkv) * kBKV > a.nk;
+    const bool partial_last = (int64_t)(jb + nkv) * C::BKV > a.nk;
     for (int j = 0; j < nkv; ++j) {
       const bool ok_j = (j == nkv - 1 && partial_last) ? step(j, std::true_type{}) : step(j, std::false_type{});
       if (!ok_j) {
@@ -390,8 +400,8 @@ acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
   }
   CUtensorMap tq, tk, tv;
   ACID_TRY(make_tmap_bf16(&tq, x.q, x.nq, x.ldq, x.ldq, kTileQ));
-  ACID_TRY(make_tmap_bf16(&tk, x.k, x.nk, x.ldk, x.ldk, kBKV));
-  ACID_TRY(make_tmap_bf16(&tv, x.v, x.nk, x.ldv, x.ldv, kBKV));
+  ACID_TRY(make_tmap_bf16(&tk, x.k, x.nk, x.ldk, x.ldk, C::BKV));
+  ACID_TRY(make_tmap_bf16(&tv, x.v, x.nk, x.ldv, x.ldv, C::BKV));
   AttnDev a;
   a.nq = x.nq;
   a.nk = x.nk;
@@ -408,13 +418,13 @@ acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
   a.part_o = nullptr;
   a.part_ml = nullptr;
   const int items = a.nqp * x.heads;
-  const int nkv_all = (int)((x.nk + kBKV - 1) / kBKV);
-  // Items fill whole waves of one CTA per SM; the items of a last, partial
-  // wave are split along the key range so that they fill one wave together,
-  // and their partial results are merged.
-  const int sms = num_sms_attn();
-  const int full = (items / sms) * sms, tail = items - full;
-  int splits = tail > 0 ? std::min(std::min(kAttnPartCtas, sms) / tail, nkv_all) : 1;
+  const int nkv_all = (int)((x.nk + C::BKV - 1) / C::BKV);
+  // Items fill whole waves of CTAS_PER_SM CTAs per SM; the items of a last,
+  // partial wave are split along the key range so that they fill one wave
+  // together, and their partial results are merged.
+  const int slots = num_sms_attn() * C::CTAS_PER_SM;
+  const int full = (items / slots) * slots, tail = items - full;
+  int splits = tail > 0 ? std::min(std::min(kAttnPartCtas, slots) / tail, nkv_all) : 1;
   const size_t part_need = (size_t)tail * splits * kBQ * (D + 2) * sizeof(float);
   const bool split_tail = full > 0 && tail > 0 && splits >= 2 && x.part != nullptr && x.part_bytes >= part_need;
   ProfScope prof(PROF_ATTENTION, 4.0 * (double)x.nq * (double)x.nk * D * x.heads, s);
