@@ -43,7 +43,7 @@ REF_SAMPLE_ROWS = 2048
 # launch, the split tail launch and the merge) per attention call of the step's
 # 1:1 self/cross mix.  Valid only for the kernel source it was measured on; any
 # other source reports null.
-ATTN_TRAFFIC = {"source_sha256_16": "7f3819367c898c87", "bytes_per_launch": (438.40e6 + 165.79e6) / 2}
+ATTN_TRAFFIC = {"source_sha256_16": "bcf60336260af114", "bytes_per_launch": (434.43e6 + 165.68e6) / 2}
 
 
 def _attn_traffic():
