@@ -103,6 +103,29 @@ def test_linear_bf16_many_row_blocks(acid, M, K, N, epi, fp32):
     assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
 
 
+@pytest.mark.parametrize("M,K,N", [(700, 192, 640), (300, 128, 1920), (513, 64, 5760), (129, 96, 160)])
+@pytest.mark.parametrize("epi", ["bias", "gelu", "gated_res", "res"])
+def test_linear_bf16_partial_last_column_tile(acid, M, K, N, epi):
+    """N not a multiple of the 256-wide tile: the last column tile reads
+    zero-filled weight rows and stores only its valid columns (CogVideoX
+    widths 1920 and 5760 among them)."""
+    rng = np.random.default_rng(M * 7 + N)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.1 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    g = rng.normal(size=N).astype(np.float32)
+    r = rng.normal(size=(M, N)).astype(np.float32)
+    has_res = epi in ("gated_res", "res")
+    res = _f32(r) if has_res else None
+    out = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), epilogue=epi, gate=_f32(g), residual=res, out=res,
+                                   out_fp32=True)
+    acc = O.linear(a, w, b)
+    ref = {"bias": acc, "gelu": O.gelu_tanh(acc), "gated_res": r + g * acc, "res": r + acc}[epi]
+    got = out.cpu().numpy()
+    tol = 2 ** -9 if epi == "gelu" else 1e-4
+    assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
+
+
 @pytest.mark.parametrize("M,K,N", [(1, 64, 64), (7, 8, 32), (127, 72, 96), (129, 200, 256), (3, 4104, 128)])
 def test_linear_bf16_edge_shapes(acid, M, K, N):
     """Single rows, K below / not a multiple of the 64-wide k-block (zero-filled
