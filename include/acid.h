@@ -68,6 +68,14 @@ const char* acid_version(void);
  * timed-out device wait: ACID_OK or ACID_ERR_TIMEOUT.  Synchronous. */
 acid_status acid_check_device_error(void);
 
+/* Diagnostic of the failure path: launches one CTA whose thread waits on an
+ * mbarrier that nothing arrives on, through the same bounded wait as the
+ * kernels but with a budget of `budget_cycles` SM clocks (1e3..1e10).  The
+ * wait runs out, raises the device flag and the kernel returns normally, so
+ * the next acid_check_device_error() reports ACID_ERR_TIMEOUT and the context
+ * stays usable.  Synchronises `stream`. */
+acid_status acid_selftest_wait_timeout(int64_t budget_cycles, acid_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Tracing: launch counting and per-launch device timing                     */
 /* ------------------------------------------------------------------------ */

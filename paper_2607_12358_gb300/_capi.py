@@ -76,6 +76,7 @@ _PROTOS = {
     "acid_last_error": (C.c_char_p, []),
     "acid_version": (C.c_char_p, []),
     "acid_check_device_error": (C.c_int, []),
+    "acid_selftest_wait_timeout": (C.c_int, [C.c_int64, _P]),
     "acid_launch_count": (C.c_int64, []),
     "acid_profile_enable": (C.c_int, [C.c_int32]),
     "acid_profile_read": (C.c_int, [C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double),

@@ -55,6 +55,12 @@ def check_device_error() -> None:
     check(load().acid_check_device_error())
 
 
+def selftest_wait_timeout(budget_cycles: int, stream=None) -> None:
+    """Runs the failure-path diagnostic (a bounded wait that runs out); the next
+    check_device_error() raises with ACID_ERR_TIMEOUT."""
+    check(load().acid_selftest_wait_timeout(int(budget_cycles), _stream(stream)))
+
+
 def launch_count() -> int:
     return int(load().acid_launch_count())
 

@@ -122,10 +122,39 @@ extern "C" const char* acid_last_error(void) { return t_last_error.c_str(); }
 
 extern "C" const char* acid_version(void) { return "acid-gb300 0.1 (sm_103a)"; }
 
+namespace acid {
+namespace {
+// One thread waits on an mbarrier that no thread arrives on, through the
+// kernels' bounded wait with a short budget: the wait runs out, raises this
+// unit's device flag and the kernel returns.
+__global__ void wait_selftest_kernel(long long limit) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) (void)mbar_wait_limit(&bar, 0, limit);
+}
+}  // namespace
+ACID_DEVICE_FLAG_READER(take_device_error_capi)
+}  // namespace acid
+
+extern "C" acid_status acid_selftest_wait_timeout(int64_t budget_cycles, acid_stream_t stream) {
+  clear_error();
+  ACID_REQUIRE(budget_cycles >= 1000 && budget_cycles <= 10000000000LL, ACID_ERR_INVALID_ARG,
+               "acid_selftest_wait_timeout: budget must be 1e3..1e10 cycles");
+  cudaStream_t s = (cudaStream_t)stream;
+  wait_selftest_kernel<<<1, 32, 0, s>>>((long long)budget_cycles);
+  ACID_CHECK_LAUNCH();
+  ACID_CUDA(cudaStreamSynchronize(s));
+  return ACID_OK;
+}
+
 extern "C" acid_status acid_check_device_error(void) {
   clear_error();
   ACID_CUDA(cudaDeviceSynchronize());
-  const unsigned int flag = take_device_error_gemm() | take_device_error_attention();
+  const unsigned int flag = take_device_error_gemm() | take_device_error_attention() | take_device_error_capi();
   if (flag) {
     set_error("a bounded device-side wait timed out");
     return ACID_ERR_TIMEOUT;

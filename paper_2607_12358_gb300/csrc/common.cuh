@@ -207,20 +207,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // About 4 s at 2 GHz: far above any legitimate wait in these kernels.
 constexpr long long kWaitLimitCycles = 8000000000LL;
 
-// Returns false (and raises the device flag) if the phase did not complete in
-// time.  Callers stop their role's loop on false.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Returns false (and raises the device flag) if the phase did not complete
+// within `limit` SM clocks.  Callers stop their role's loop on false.
+__device__ __forceinline__ bool mbar_wait_limit(uint64_t* bar, uint32_t parity, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     #pragma unroll 1
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (clock64() - t0 > kWaitLimitCycles) {
+    if (clock64() - t0 > limit) {
       atomicExch(&g_device_error, 1u);
       return false;
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  return mbar_wait_limit(bar, parity, kWaitLimitCycles);
 }
 
 // ---------------------------------------------------------------------------

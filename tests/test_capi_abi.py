@@ -109,6 +109,8 @@ def test_host_validation_without_gpu(lib):
     assert lib.acid_drift_signal(None, None, 10, 7, None, None, None, 0, None) == A.ACID_ERR_INVALID_ARG
     assert lib.acid_cache_apply(None, None, None, 10, A.ACID_BF16, None) == A.ACID_ERR_INVALID_ARG
     assert lib.acid_cache_apply(None, None, None, 0, A.ACID_BF16, None) == A.ACID_OK
+    # the failure-path diagnostic validates its budget before launching anything
+    assert lib.acid_selftest_wait_timeout(10, None) == A.ACID_ERR_INVALID_ARG
     assert lib.acid_linear_forward(A.ACID_BF16, None, 64, 10, 64, None, None, 64, None, 64, 9, None, None, 0, 0,
                                    None) == A.ACID_ERR_INVALID_ARG
     assert lib.acid_attention_forward(A.ACID_BF16, None, 64, None, 64, None, 64, None, 64, 0, 4, 1, 64,
