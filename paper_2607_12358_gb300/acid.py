@@ -363,6 +363,29 @@ class Loop:
                                        _stream(self.stream)))
         return lg if log else None
 
+    def checkpoint(self) -> dict:
+        """The generation's resumable state: a copy of the controller struct and
+        of the loop workspace (caches, text context, RoPE table).  Together with
+        the latent it restores the generation exactly (Loop.restore)."""
+        st = A.acid_loop_state()
+        C.memmove(C.byref(st), C.byref(self.state), C.sizeof(st))
+        n = self.model.workspace_size()
+        off = self.ws_ptr - self.ws.data_ptr()
+        return {"state": st, "workspace": self.ws[off:off + n].clone()}
+
+    @classmethod
+    def restore(cls, model: DeviceModel, cfg_struct, ckpt: dict, device="cuda", stream=None) -> "Loop":
+        """A Loop that continues a checkpointed generation in a fresh workspace."""
+        obj = cls.__new__(cls)
+        obj.model, obj.cfg, obj.text, obj.stream = model, cfg_struct, None, stream
+        obj.ws, obj.ws_ptr, obj.ws_bytes = _aligned_ws(model.workspace_size(), device)
+        n = ckpt["workspace"].numel()
+        off = obj.ws_ptr - obj.ws.data_ptr()
+        obj.ws[off:off + n].copy_(ckpt["workspace"])
+        obj.state = A.acid_loop_state()
+        C.memmove(C.byref(obj.state), C.byref(ckpt["state"]), C.sizeof(obj.state))
+        return obj
+
 
 def log_to_dict(lg: A.acid_step_log) -> dict:
     return {k: getattr(lg, k) for k, _ in A.acid_step_log._fields_}

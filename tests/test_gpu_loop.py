@@ -134,6 +134,37 @@ def test_toy_loop_transition_schedule(acid, k):
     assert [l["tau"] for l in logs[cfg.warmup:]] == sched[cfg.warmup:]
 
 
+@pytest.mark.parametrize("method", ["teacache", "easycache", "dicache"])
+def test_checkpoint_resume_is_exact(acid, method):
+    """A generation stopped after k steps, checkpointed (controller struct and
+    loop workspace), dropped and restored into a fresh workspace continues bit
+    for bit like an uninterrupted one."""
+    over = dict(method="easycache", tau_low=0.02, tau_high=0.04) if method == "easycache" else {}
+    cfg = S.get_config("toy", steps=10, **over)
+    w = S.model_weights(cfg, 17)
+    lat = S.latent(cfg, 17)
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg, method=method)
+    ref = torch.from_numpy(lat).to(DEV)
+    full = acid.Loop(model, c, None, DEV)
+    ref_logs = [acid.log_to_dict(full.step(ref)) for _ in range(cfg.steps)]
+    x = torch.from_numpy(lat).to(DEV)
+    part = acid.Loop(model, c, None, DEV)
+    logs = [acid.log_to_dict(part.step(x)) for _ in range(6)]
+    ckpt = part.checkpoint()
+    x_saved = x.clone()
+    del part
+    torch.cuda.synchronize()
+    resumed = acid.Loop.restore(model, c, ckpt, DEV)
+    logs += [acid.log_to_dict(resumed.step(x_saved)) for _ in range(cfg.steps - 6)]
+    acid.check_device_error()
+    np.testing.assert_array_equal(x_saved.cpu().numpy(), ref.cpu().numpy())
+    for a, b in zip(logs, ref_logs):
+        assert a["computed"] == b["computed"]
+        assert (a["signal"] != a["signal"] and b["signal"] != b["signal"]) or a["signal"] == b["signal"]
+    assert 0 < sum(l["computed"] for l in logs) < cfg.steps
+
+
 def test_toy_loop_forced_decisions(acid):
     cfg = S.get_config("toy", steps=6)
     w = S.model_weights(cfg, 3)
