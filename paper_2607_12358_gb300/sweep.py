@@ -190,6 +190,9 @@ def main(argv=None):
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--host-loop", action="store_true", help="host-driven loop instead of the CUDA graph")
     ap.add_argument("--out", default=None, help="write the JSON here (default: stdout)")
+    ap.add_argument("--jsonl", default=None,
+                    help="also write one JSON line per run and step (run, step, t, signal, dsignal, tau, sigma, "
+                         "computed)")
     a = ap.parse_args(argv)
 
     import acid_synth as S
@@ -207,6 +210,13 @@ def main(argv=None):
     res = sweep(cfg, weights, S.latent(cfg, a.seed), text, tau_low=a.tau_low, tau_high=a.tau_high,
                 transitions=a.transitions, deltas=a.deltas, method=a.method, graph=not a.host_loop)
     out = json.dumps(res)
+    if a.jsonl:
+        with open(a.jsonl, "w") as f:
+            for r in [res["full"], res["fixed_low"], res["fixed_high"]] + res["runs"]:
+                for i in range(r["steps"]):
+                    f.write(json.dumps({"run": r["name"], "step": i, "signal": r["signal"][i],
+                                        "dsignal": r["dsignal"][i], "tau": r["tau"][i],
+                                        "computed": r["decisions"][i]}) + "\n")
     if a.out:
         with open(a.out, "w") as f:
             f.write(out + "\n")
