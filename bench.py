@@ -62,6 +62,25 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(value: float, world: int) -> float:
+    """The largest `value` over all ranks: the job takes as long as its slowest
+    rank (the process group must be initialised when world > 1)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(value)], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.item()
+
+
+def job_rate(steps: int, seconds: float, world: int) -> float:
+    """Whole-job steps/s: each of the `world` replicas runs `steps` steps in at
+    most `seconds` (the max over ranks)."""
+    return world * steps / seconds
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -264,12 +283,8 @@ def run_ours(args) -> None:
     acid.profile_enable(False)
     acid.check_device_error()
     assert torch.isfinite(lat).all().item()
-    t_max = ms
-    if world > 1:
-        tt = torch.tensor([ms], dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        t_max = tt.item()
-    value = world * K / (t_max / 1000.0)
+    t_max = max_over_ranks(ms, world)
+    value = job_rate(K, t_max / 1000.0, world)
 
     # ---- end to end: latent from pinned host memory each step, result read back
     c2, keep2 = acid.loop_cfg(cfg, n_steps=W + K + 1, tau_low=-1.0, tau_high=-1.0)
@@ -288,11 +303,7 @@ def run_ours(args) -> None:
         loop2.step(dlat, log=False)
         host_out.copy_(dlat, non_blocking=True)
     barrier()
-    e2e_s = time.perf_counter() - t0
-    if world > 1:
-        tt = torch.tensor([e2e_s], dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = tt.item()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
     lat_bytes = host_in.numel() * 4
 
     # ---- the workload's own thresholds (effective rate under caching)
@@ -316,7 +327,7 @@ def run_ours(args) -> None:
     t0 = time.perf_counter()
     acid.acid_denoise_loop(model, c4, lat4, text, log=False, graph=True)
     barrier()
-    graph_s = time.perf_counter() - t0
+    graph_s = max_over_ranks(time.perf_counter() - t0, world)
     acid.check_device_error()
 
     if rank != 0:
@@ -345,10 +356,10 @@ def run_ours(args) -> None:
         "acid_mode": {"steps_per_s": K / (acid_ms / 1000.0), "computed_steps": computed, "of": K,
                       "tau_low": cfg.tau_low, "tau_high": cfg.tau_high, "delta": cfg.delta,
                       "note": "random weights: the skip rate says nothing about a trained model"},
-        "graph_mode": {"steps_per_s": world * K / graph_s,
+        "graph_mode": {"steps_per_s": job_rate(K, graph_s, world),
                        "note": "the same K steps, every step computed, as one CUDA graph (WHILE over steps, "
                                "IF/ELSE per decision); wall time including graph build and instantiation"},
-        "e2e": {"value": world * K / e2e_s, "unit": UNIT, "h2d_bytes_per_step": lat_bytes,
+        "e2e": {"value": job_rate(K, e2e_s, world), "unit": UNIT, "h2d_bytes_per_step": lat_bytes,
                 "d2h_bytes_per_step": lat_bytes},
         "gpu_launches": launches,
         "clocks": clk.summary(),
