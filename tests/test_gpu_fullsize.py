@@ -200,3 +200,30 @@ def test_cog_easycache_step_signal(acid):
     assert abs(logs[2]["signal"] - s_ref) <= 1e-3 * s_ref, (logs[2]["signal"], s_ref)
     skip, tau, sg, _ = O.AcidController(cfg.tau_low, cfg.tau_high, cfg.delta).step(logs[2]["signal"])
     assert bool(logs[2]["computed"]) == (not skip)
+
+
+def test_wan_full_model_graph_equals_host_loop(acid):
+    """The whole 30-block Wan model for four steps with its own thresholds:
+    one CUDA graph (signal and Algorithm 1 on the device) and the host-driven
+    loop run the same kernels, so the latents are bit-identical and every
+    logged signal and decision agrees."""
+    cfg = S.get_config("wan")
+    w = S.model_weights(cfg, 22)
+    model = acid.DeviceModel(cfg, w, DEV)
+    del w
+    text = torch.from_numpy(S.text(cfg, 22)).to(DEV, torch.bfloat16)
+    lat = S.latent(cfg, 22)
+    outs = []
+    for graph in (False, True):
+        c, keep = acid.loop_cfg(cfg, n_steps=4)
+        x = torch.from_numpy(lat).to(DEV)
+        logs = acid.acid_denoise_loop(model, c, x, text, graph=graph)
+        acid.check_device_error()
+        outs.append((x.cpu().numpy(), logs))
+    (xa, la), (xb, lb) = outs
+    np.testing.assert_array_equal(xa, xb)
+    for a, b in zip(la, lb):
+        assert a["computed"] == b["computed"]
+        for k in ("signal", "dsignal", "tau", "sigma"):
+            assert (a[k] != a[k] and b[k] != b[k]) or a[k] == b[k], (k, a, b)
+    assert np.isfinite(xa).all()
