@@ -193,6 +193,9 @@ acid_status acid_attention_forward(int32_t dtype, const void* q, int64_t ldq, co
                                    int64_t ldk, const void* v, int64_t ldv, void* out, int64_t ldo,
                                    int64_t nq, int64_t nk, int32_t heads, int32_t head_dim,
                                    void* workspace, size_t workspace_bytes, acid_stream_t stream);
+/* Bytes of the optional acid_attention_forward workspace for head_dim (the
+ * partial results of a split last wave: kept for 160 CTAs of 256 rows, fp32
+ * output rows plus the running max and sum). */
 acid_status acid_attention_workspace_size(int32_t head_dim, size_t* bytes);
 
 /* adaLN LayerNorm: y = LN(x) * (1 + scale) + shift per row of x [rows, d]
