@@ -175,7 +175,8 @@ typedef enum {
  *   gate       fp32 [N] (ACID_EPI_GATED_RES), residual [M, N] row stride ldr
  *              in the output dtype (may equal out: in place).
  * bf16 runs on tcgen05 (fp32 accumulation): N % 32 == 0, K % 8 == 0, rows
- * 16-byte aligned.  fp32 runs on the FP32 pipes: N even. */
+ * 16-byte aligned.  fp32 runs on the FP32 pipes: N even.  M = 0 returns
+ * ACID_OK without a launch (the pointers may then be NULL). */
 acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t lda, int64_t M, int32_t K,
                                 const void* W, const float* bias, int32_t N, void* out, int64_t ldo,
                                 int32_t epilogue, const float* gate, const void* residual,
@@ -183,7 +184,8 @@ acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t lda, int64
 
 /* Multi-head attention softmax(q k^T / sqrt(head_dim)) v, per head h reading
  * columns [h*head_dim, (h+1)*head_dim) of q (row stride ldq), k (ldk), v (ldv)
- * and writing the same columns of out (ldo).  nq, nk >= 1 rows.  bf16 runs on
+ * and writing the same columns of out (ldo).  nk >= 1 key rows; nq = 0
+ * returns ACID_OK without a launch (q and out may then be NULL).  bf16 runs on
  * tcgen05 with head_dim 64 or 128; fp32 with head_dim a multiple of 32, <= 128.
  *   workspace  optional (NULL, 0): device scratch of
  *              acid_attention_workspace_size bytes.  With it, the work that

@@ -492,9 +492,9 @@ __global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__
 }  // namespace
 
 acid_status attention_forward(int dtype, const AttnArgs& x, cudaStream_t s) {
-  ACID_REQUIRE(x.q && x.k && x.v && x.out, ACID_ERR_INVALID_ARG, "attention: null pointer");
   ACID_REQUIRE(x.nk > 0 && x.nq >= 0 && x.heads > 0, ACID_ERR_INVALID_ARG, "attention: bad shape");
-  if (x.nq == 0) return ACID_OK;
+  if (x.nq == 0) return ACID_OK;  // no query rows: nothing is read, pointers may be null
+  ACID_REQUIRE(x.q && x.k && x.v && x.out, ACID_ERR_INVALID_ARG, "attention: null pointer");
   if (dtype == ACID_FP32) {
     ACID_REQUIRE(x.head_dim % 32 == 0 && x.head_dim <= 128, ACID_ERR_UNSUPPORTED,
                  "attention fp32: head_dim must be 32, 64, 96 or 128");

@@ -233,7 +233,7 @@ extern "C" acid_status acid_attention_forward(int32_t dtype, const void* q, int6
   const int64_t w = (int64_t)heads * head_dim;
   ACID_REQUIRE(ldq >= w && ldk >= w && ldv >= w && ldo >= w, ACID_ERR_INVALID_ARG,
                "acid_attention_forward: row stride smaller than heads * head_dim");
-  ACID_REQUIRE(nq >= 1 && nk >= 1, ACID_ERR_INVALID_ARG, "acid_attention_forward: nq and nk must be >= 1");
+  ACID_REQUIRE(nq >= 0 && nk >= 1, ACID_ERR_INVALID_ARG, "acid_attention_forward: need nq >= 0 and nk >= 1");
   AttnArgs a;
   a.q = q; a.ldq = ldq;
   a.k = k; a.ldk = ldk;

@@ -568,10 +568,10 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__
 
 acid_status linear_forward_f32(const void* A, int64_t lda, int64_t M, int K, int w_dtype, const void* W, int N,
                                void* out, int64_t ldo, const Epilogue& epi, cudaStream_t s) {
-  ACID_REQUIRE(A && W && out, ACID_ERR_INVALID_ARG, "linear: null pointer");
   ACID_REQUIRE(M >= 0 && K > 0 && N > 0, ACID_ERR_INVALID_ARG, "linear: bad shape");
+  if (M == 0) return ACID_OK;  // no rows: nothing is read, pointers may be null
+  ACID_REQUIRE(A && W && out, ACID_ERR_INVALID_ARG, "linear: null pointer");
   ACID_REQUIRE(N % 2 == 0, ACID_ERR_UNSUPPORTED, "linear fp32: N must be even");
-  if (M == 0) return ACID_OK;
   dim3 grid((N + SB - 1) / SB, (unsigned)((M + SB - 1) / SB));
   if (w_dtype == ACID_BF16)
     gemm_f32_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(static_cast<const float*>(A), lda, M, K,
@@ -587,9 +587,9 @@ acid_status linear_forward_f32(const void* A, int64_t lda, int64_t M, int K, int
 
 acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out,
                            int64_t ldo, const Epilogue& epi, cudaStream_t s) {
-  ACID_REQUIRE(A && W && out, ACID_ERR_INVALID_ARG, "linear: null pointer");
   ACID_REQUIRE(M >= 0 && K > 0 && N > 0, ACID_ERR_INVALID_ARG, "linear: bad shape");
-  if (M == 0) return ACID_OK;
+  if (M == 0) return ACID_OK;  // no rows: nothing is read, pointers may be null
+  ACID_REQUIRE(A && W && out, ACID_ERR_INVALID_ARG, "linear: null pointer");
   ACID_REQUIRE(epi.kind != EPI_ROPE_QKV || (epi.rope.table != nullptr && epi.head_dim > 0 && epi.d > 0),
                ACID_ERR_INVALID_ARG, "linear: RoPE epilogue needs a table");
   ACID_REQUIRE(epi.kind != EPI_ROPE_QKV ||

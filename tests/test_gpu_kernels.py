@@ -241,3 +241,22 @@ def test_layernorm_mod(acid, d):
     assert np.abs(got - ref).max() <= 1e-4 * (1 + np.abs(ref).max())
     got16 = acid.acid_layernorm_mod(_bf(x), _f32(sh), _f32(sc)).float().cpu().numpy()
     assert np.abs(got16 - ref).max() <= 2 ** -8 * (1 + np.abs(ref).max())
+
+
+def test_empty_inputs_return_without_launching(acid):
+    """Zero rows: the linear layer, attention, LayerNorm-mod and cache apply
+    return OK and launch nothing."""
+    n0 = acid.launch_count()
+    a = torch.empty(0, 128, dtype=torch.bfloat16, device=DEV)
+    w = torch.zeros(256, 128, dtype=torch.bfloat16, device=DEV)
+    assert acid.acid_linear_forward(a, w).shape == (0, 256)
+    q = torch.empty(0, 256, dtype=torch.bfloat16, device=DEV)
+    kv = torch.zeros(64, 256, dtype=torch.bfloat16, device=DEV)
+    assert acid.acid_attention_forward(q, kv, kv, 2).shape == (0, 256)
+    x = torch.empty(0, 256, dtype=torch.bfloat16, device=DEV)
+    assert acid.acid_layernorm_mod(x).shape[0] == 0
+    e = torch.empty(0, dtype=torch.bfloat16, device=DEV)
+    acid.acid_cache_apply(e, e, out=e)
+    torch.cuda.synchronize()
+    acid.check_device_error()
+    assert acid.launch_count() == n0
