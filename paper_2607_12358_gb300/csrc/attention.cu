@@ -3,9 +3,9 @@
 // token by the QKV projection's epilogue, so this kernel reads pre-rotated
 // operands.
 //
-// bf16 path: a flash-attention kernel on tcgen05 tensor cores.  One CTA owns
-// two 128-row query tiles (a, b) of one head and streams 128-key K/V tiles
-// that both query tiles share:
+// bf16 path: a flash-attention kernel on tcgen05 tensor cores.  A work item
+// is two 128-row query tiles (a, b) of one head; its CTA streams 128-key K/V
+// tiles that both query tiles share:
 //   warp 0      TMA producer: Q_a, Q_b once, then K_j and V_j into 2-deep rings
 //               (128-byte swizzle);
 //   warp 1      MMA issuer, in the order S_a(0) S_b(0) | PV_a(j) S_a(j+1)
@@ -19,6 +19,11 @@
 //               in TMEM only when the running max grows by more than 2^8 (the
 //               final division by the sum makes the result independent of
 //               when rescaling happens).
+// attn_tc_kernel runs one item per CTA (long key ranges: self and joint
+// attention).  attn_persist_kernel runs items of a few key tiles (cross
+// attention over a short text) on persistent CTAs: the next item's Q loads
+// and first S MMAs overlap the current item's last softmax, and the output
+// leaves through shared memory and TMA stores.
 // fp32 path: one warp per query row, exact expf, for the fp32 mode.
 #include <cudaTypedefs.h>
 #include <math.h>
@@ -31,6 +36,8 @@
 namespace acid {
 
 acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows);
+acid_status make_tmap_bf16_box(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                               int box_cols, int box_rows, CUtensorMapSwizzle swizzle);
 
 namespace {
 
@@ -47,12 +54,14 @@ struct AttnDev {
   int64_t ldo;
   int o_col;
   float scale_log2;  // log2(e) / sqrt(head_dim)
-  // work item = (query-tile pair, head), numbered head-major; CTA blockIdx.x
-  // handles item item_base + blockIdx.x / splits and the split-th part of the
-  // key range.  With splits > 1 the CTA writes its unnormalised output and
-  // (max, sum) per row to part_o / part_ml instead of the final output.
+  // work item = (query-tile pair, head), numbered head-major.  attn_tc_kernel:
+  // CTA blockIdx.x handles item item_base + blockIdx.x / splits and the
+  // split-th part of the key range; with splits > 1 it writes its
+  // unnormalised output and (max, sum) per row to part_o / part_ml instead of
+  // the final output.  attn_persist_kernel: CTA blockIdx.x handles items
+  // item_base + blockIdx.x + k * gridDim.x below item_end.
   int nqp;
-  int item_base;
+  int item_base, item_end;
   int splits;
   float* part_o;   // [CTA][256 rows][D]
   float* part_ml;  // [CTA][256 rows][2]
@@ -77,12 +86,114 @@ struct AttnCfg {
   static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
   static constexpr int OFF_BAR = OFF_V + 2 * KV_BYTES;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  // attn_persist_kernel adds the output staging: per softmax warp two
+  // 32-row x 32-column bf16 boxes (64-byte swizzle) for TMA stores
+  static constexpr int STAGE_BOX = 32 * 64;
+  static constexpr int OFF_STAGE_P = OFF_V + 2 * KV_BYTES;
+  static constexpr int OFF_BAR_P = OFF_STAGE_P + 8 * 2 * STAGE_BOX;
+  static constexpr int SMEM_P = OFF_BAR_P + 256 + 1024;
   // TMEM columns: S_a [0,BKV), S_b [BKV,2BKV) (P_t over the first BKV/2
   // columns of S_t), O_a [2BKV, 2BKV+D), O_b [2BKV+D, 2BKV+2D)
   static constexpr uint32_t S_COL = 0, O_COL = 2 * BKV;
   static constexpr uint32_t TMEM_COLS = 2 * BKV + 2 * D;
   __host__ __device__ static constexpr uint32_t o_col(int t) { return O_COL + t * D; }
 };
+
+// Softmax of one key tile for this thread's query row (row r of tile t is
+// TMEM lane r): waits for S_t, writes P_t = 2^(s * scale - m) over the S
+// region as bf16 pairs, updates the running reference max m and sum l,
+// rescales O_t when the reference moves, and hands P_t to the MMA warp.
+// phase: this tile's step count in the CTA (barrier parity); first: the
+// item's first key tile; valid: keys of a masked (partial last) tile.
+template <int D, bool MASKED>
+__device__ __forceinline__ bool softmax_tile(uint64_t* s_full, uint64_t* pv_done, uint64_t* p_full, int phase,
+                                             bool first, int valid, uint32_t s_addr, uint32_t o_addr,
+                                             float scale_log2, float& m_run, float& l_run) {
+  using C = AttnCfg<D>;
+  if (!mbar_wait(s_full, phase & 1)) return false;
+  // consume pv_done phase - 1 (already complete: s_full(phase) is committed
+  // after PV(phase - 1)) so that no later parity wait is two phases behind;
+  // at an item's first tile the previous item's output pass consumed it
+  if (!first && !mbar_wait(pv_done, (phase - 1) & 1)) return false;
+  tc_fence_after();
+  float s[C::BKV];
+#pragma unroll
+  for (int c = 0; c < C::BKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
+  tmem_wait_ld();
+  bool resc = false;
+  float f = 1.0f;
+  if constexpr (MASKED) {
+#pragma unroll
+    for (int i = 0; i < C::BKV; ++i)
+      if (i >= valid) s[i] = -INFINITY;
+  }
+  // e = s * scale - m_run in place (packed pairs; the first tile uses 0 as
+  // the reference), with the row max of e alongside in four independent
+  // 3-input max chains on the ALU pipe.  s_full(phase) is committed after
+  // PV(phase - 1), so O_t and the P_t region are free here.  Lazy rescaling:
+  // the reference max moves only on the first tile or when the row max
+  // exceeds it by more than 2^8; then e is shifted in place.
+  const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
+  {
+    const float mref = first ? 0.f : m_run;
+    const uint64_t nm2 = f2_pack(-mref, -mref);
+    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+    for (int i = 0; i < C::BKV / 2; ++i) {
+      f2_unpack(f2_fma(f2_pack(s[2 * i], s[2 * i + 1]), sc2, nm2), s[2 * i], s[2 * i + 1]);
+      m4[i & 3] = fmax3(m4[i & 3], s[2 * i], s[2 * i + 1]);
+    }
+    const float me = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+    if (first || me > kRescaleLog2) {
+      if (!first) {
+        resc = true;
+        f = ex2_approx(-me);
+        l_run *= f;
+      }
+      m_run = mref + me;
+      const uint64_t sh2 = f2_pack(-me, -me);
+#pragma unroll
+      for (int i = 0; i < C::BKV / 2; ++i) f2_unpack(f2_add(f2_pack(s[2 * i], s[2 * i + 1]), sh2), s[2 * i], s[2 * i + 1]);
+    }
+  }
+  // P = 2^e as bf16 pairs over the first BKV/2 columns of S_t, with the row
+  // sum as packed fp32 pairs
+  uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
+#pragma unroll
+  for (int half = 0; half < C::BKV / 64; ++half) {
+    uint32_t pk[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const float p0 = ex2_approx(s[half * 64 + 2 * i]), p1 = ex2_approx(s[half * 64 + 2 * i + 1]);
+      if (i & 1)
+        acc1 = f2_add(acc1, f2_pack(p0, p1));
+      else
+        acc0 = f2_add(acc0, f2_pack(p0, p1));
+      pk[i] = pack_bf16(p0, p1);
+    }
+    tmem_st32(s_addr + half * 32, pk);
+  }
+  float a0, a1, b0, b1;
+  f2_unpack(acc0, a0, a1);
+  f2_unpack(acc1, b0, b1);
+  const float ls = (a0 + a1) + (b0 + b1);
+  l_run += ls;
+  if (__any_sync(0xffffffffu, resc)) {
+#pragma unroll 1
+    for (int c = 0; c < D; c += 32) {
+      uint32_t o[32];
+      tmem_ld32(o_addr + c, o);
+      tmem_wait_ld();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+      tmem_st32(o_addr + c, o);
+    }
+  }
+  tmem_wait_st();
+  tc_fence_before();
+  mbar_arrive(p_full);
+  return true;
+}
 
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
@@ -220,89 +331,9 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
     // One key tile; the masked variant (keys past the end of the sequence)
     // is compiled separately and runs only on a partial last tile.
     auto step = [&](int j, auto masked) -> bool {
-      if (!mbar_wait(&s_full[t], j & 1)) return false;
-      // consume pv_done_t phase j-1 (already complete: s_full_t(j) is committed
-      // after PV_t(j-1)) so that the final parity wait is never two phases ahead
-      if (j > 0 && !mbar_wait(&pv_done[t], (j - 1) & 1)) return false;
-      tc_fence_after();
-      float s[C::BKV];
-#pragma unroll
-      for (int c = 0; c < C::BKV / 32; ++c) tmem_ld32(s_addr + c * 32, reinterpret_cast<uint32_t*>(s + c * 32));
-      tmem_wait_ld();
-      bool resc = false;
-      float f = 1.0f;
-      if constexpr (decltype(masked)::value) {
-        const int valid = (int)(a.nk - (int64_t)(jb + j) * C::BKV);  // keys of the last tile
-#pragma unroll
-        for (int i = 0; i < C::BKV; ++i)
-          if (i >= valid) s[i] = -INFINITY;
-      }
-      // e = s * scale - m_run in place (packed pairs; the first tile uses 0 as
-      // the reference), with the row max of e alongside in four independent
-      // 3-input max chains on the ALU pipe.  s_full_t(j) is committed after
-      // PV_t(j-1), so O_t and the P_t region are free here.  Lazy rescaling:
-      // the reference max moves only on the first tile or when the row max
-      // exceeds it by more than 2^8; then e is shifted in place.
-      const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2);
-      {
-        const float mref = j == 0 ? 0.f : m_run;
-        const uint64_t nm2 = f2_pack(-mref, -mref);
-        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-        for (int i = 0; i < C::BKV / 2; ++i) {
-          f2_unpack(f2_fma(f2_pack(s[2 * i], s[2 * i + 1]), sc2, nm2), s[2 * i], s[2 * i + 1]);
-          m4[i & 3] = fmax3(m4[i & 3], s[2 * i], s[2 * i + 1]);
-        }
-        const float me = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-        if (j == 0 || me > kRescaleLog2) {
-          if (j > 0) {
-            resc = true;
-            f = ex2_approx(-me);
-            l_run *= f;
-          }
-          m_run = mref + me;
-          const uint64_t sh2 = f2_pack(-me, -me);
-#pragma unroll
-          for (int i = 0; i < C::BKV / 2; ++i) f2_unpack(f2_add(f2_pack(s[2 * i], s[2 * i + 1]), sh2), s[2 * i], s[2 * i + 1]);
-        }
-      }
-      // P = 2^e as bf16 pairs over the first 64 columns of S_t, with the row
-      // sum as packed fp32 pairs
-      uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
-#pragma unroll
-      for (int half = 0; half < C::BKV / 64; ++half) {
-        uint32_t pk[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float p0 = ex2_approx(s[half * 64 + 2 * i]), p1 = ex2_approx(s[half * 64 + 2 * i + 1]);
-          if (i & 1)
-            acc1 = f2_add(acc1, f2_pack(p0, p1));
-          else
-            acc0 = f2_add(acc0, f2_pack(p0, p1));
-          pk[i] = pack_bf16(p0, p1);
-        }
-        tmem_st32(s_addr + half * 32, pk);
-      }
-      float a0, a1, b0, b1;
-      f2_unpack(acc0, a0, a1);
-      f2_unpack(acc1, b0, b1);
-      const float ls = (a0 + a1) + (b0 + b1);
-      l_run += ls;
-      if (__any_sync(0xffffffffu, resc)) {
-#pragma unroll 1
-        for (int c = 0; c < D; c += 32) {
-          uint32_t o[32];
-          tmem_ld32(o_addr + c, o);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
-          tmem_st32(o_addr + c, o);
-        }
-      }
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(&p_full[t]);
-          return true;
+      return softmax_tile<D, decltype(masked)::value>(&s_full[t], &pv_done[t], &p_full[t], j, j == 0,
+                                                      (int)(a.nk - (int64_t)(jb + j) * C::BKV), s_addr, o_addr,
+                                                      a.scale_log2, m_run, l_run);
     };
     const bool partial_last = (int64_t)(jb + nkv) * C::BKV > a.nk;
     for (int j = 0; j < nkv; ++j) {
@@ -341,6 +372,228 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
     if (a.splits > 1 && ok && row < a.nq)
       *reinterpret_cast<float2*>(a.part_ml + ((int64_t)blockIdx.x * kBQ + t * kTileQ + r) * 2) =
           make_float2(m_run, l_run);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// Persistent variant for items of a few key tiles.  Each CTA walks the items
+// item_base + blockIdx.x + k * gridDim.x; one counter g numbers its key-tile
+// steps across items, and every per-step barrier phase and ring slot follows
+// it.  Q_t of the next item is loaded once the current item's last S_t MMA
+// has completed (q_empty), so the MMA warp issues the next item's first S
+// right after the current item's last PV.  The output leaves through two
+// staging boxes per softmax warp and TMA stores, which frees the softmax
+// warps for the next item.
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
+    attn_persist_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                        AttnDev a) {
+  using C = AttnCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint8_t* sK = smem + C::OFF_K;
+  uint8_t* sV = smem + C::OFF_V;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR_P);
+  uint64_t* q_full = bars + 0;    // [2] per query tile
+  uint64_t* q_empty = bars + 2;   // [2] per query tile
+  uint64_t* k_full = bars + 4;    // [2]
+  uint64_t* k_empty = bars + 6;   // [2]
+  uint64_t* v_full = bars + 8;    // [2]
+  uint64_t* v_empty = bars + 10;  // [2]
+  uint64_t* s_full = bars + 12;   // [2] per query tile
+  uint64_t* p_full = bars + 14;   // [2] per query tile
+  uint64_t* pv_done = bars + 16;  // [2] per query tile
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int item0 = a.item_base + (int)blockIdx.x, item_step = (int)gridDim.x;
+  const int n_items = item0 < a.item_end ? (a.item_end - 1 - item0) / item_step + 1 : 0;
+  const int nkv = (int)((a.nk + C::BKV - 1) / C::BKV);
+  const int total = n_items * nkv;  // key-tile steps of this CTA
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+    tma_prefetch_desc(&tmO);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&q_full[i], 1);
+      mbar_init(&q_empty[i], 1);
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&v_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], 128);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------------------------------- TMA producer
+      bool ok = true;
+      for (int k = 0, g = 0; ok && k < n_items; ++k) {
+        const int item = item0 + k * item_step;
+        const int qt = item % a.nqp, h = item / a.nqp;
+        // Q_t of item k replaces Q_t of item k - 1 once that item's last S_t is done
+        for (int t = 0; t < 2 && ok; ++t) {
+          if (k > 0 && !mbar_wait(&q_empty[t], (k - 1) & 1)) { ok = false; break; }
+          mbar_expect_tx(&q_full[t], C::T_BYTES);
+          for (int c = 0; c < C::CH; ++c)
+            tma_load_2d(sQ + t * C::T_BYTES + c * C::CHUNK_Q, &tmQ, &q_full[t], a.q_col + h * D + c * 64,
+                        qt * kBQ + t * kTileQ);
+        }
+        for (int j = 0; ok && j < nkv; ++j, ++g) {
+          const int st = g & 1, round = g >> 1;
+          if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) { ok = false; break; }
+          mbar_expect_tx(&k_full[st], C::KV_BYTES);
+          for (int c = 0; c < C::CH; ++c)
+            tma_load_2d(sK + st * C::KV_BYTES + c * C::CHUNK_KV, &tmK, &k_full[st], a.k_col + h * D + c * 64,
+                        j * C::BKV);
+          if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) { ok = false; break; }
+          mbar_expect_tx(&v_full[st], C::KV_BYTES);
+          for (int c = 0; c < C::CH; ++c)
+            tma_load_2d(sV + st * C::KV_BYTES + c * C::CHUNK_KV, &tmV, &v_full[st], a.v_col + h * D + c * 64,
+                        j * C::BKV);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---------------------------------------- MMA issuer
+      constexpr uint32_t idesc_s = idesc_bf16_f32(128, C::BKV, false, false);
+      constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
+      const uint64_t qdesc = smem_desc_sw128(smem_u32(sQ), 16, 1024);
+      const uint64_t kdesc = smem_desc_sw128(smem_u32(sK), 16, 1024);
+      const uint64_t vdesc = smem_desc_sw128(smem_u32(sV), C::CHUNK_KV, 1024);
+      // S_t = Q_t K^T of step g into the S region of tile t; after an item's
+      // last key tile (last_tile) the producer may replace Q_t
+      auto issue_s = [&](int t, int g, bool last_tile) {
+        const uint64_t a0 = qdesc + (uint64_t)((t * C::T_BYTES) >> 4);
+        const uint64_t b0 = kdesc + (uint64_t)(((g & 1) * C::KV_BYTES) >> 4);
+        const uint32_t d = tmem + C::S_COL + t * C::BKV;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t off_a = (uint64_t)(((kk >> 2) * C::CHUNK_Q + (kk & 3) * 32) >> 4);
+          const uint64_t off_b = (uint64_t)(((kk >> 2) * C::CHUNK_KV + (kk & 3) * 32) >> 4);
+          mma_bf16_ss(d, a0 + off_a, b0 + off_b, idesc_s, kk != 0);
+        }
+        mma_commit(&s_full[t]);
+        if (last_tile) mma_commit(&q_empty[t]);
+      };
+      bool ok = total > 0 && mbar_wait(&k_full[0], 0);
+      for (int t = 0; t < 2 && ok; ++t) {
+        if (!mbar_wait(&q_full[t], 0)) { ok = false; break; }
+        tc_fence_after();
+        issue_s(t, 0, nkv == 1);
+      }
+      if (ok) mma_commit(&k_empty[0]);
+      // step g (key tile j of item k): PV_a(g) S_a(g+1) PV_b(g) S_b(g+1); at an
+      // item boundary S(g+1) reads the next item's Q
+      for (int g = 0, j = 0, k = 0; ok && g < total; ++g) {
+        const int st = g & 1, gn = g + 1;
+        const bool boundary = j + 1 == nkv;  // step gn starts item k + 1
+        const int jn = boundary ? 0 : j + 1;
+        for (int t = 0; t < 2 && ok; ++t) {
+          if (!mbar_wait(&p_full[t], g & 1)) { ok = false; break; }
+          if (t == 0 && !mbar_wait(&v_full[st], (g >> 1) & 1)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t b0 = vdesc + (uint64_t)((st * C::KV_BYTES) >> 4);
+          const uint32_t d = tmem + C::o_col(t), p0 = tmem + C::S_COL + t * C::BKV;
+#pragma unroll
+          for (int kk = 0; kk < C::BKV / 16; ++kk)
+            mma_bf16_ts(d, p0 + kk * 8, b0 + (uint64_t)((kk * 16 * 128) >> 4), idesc_o, (j | kk) != 0);
+          mma_commit(&pv_done[t]);
+          if (t == 1) mma_commit(&v_empty[st]);
+          if (gn < total) {
+            if (t == 0 && !mbar_wait(&k_full[st ^ 1], (gn >> 1) & 1)) { ok = false; break; }
+            if (boundary && !mbar_wait(&q_full[t], (k + 1) & 1)) { ok = false; break; }
+            tc_fence_after();
+            issue_s(t, gn, jn == nkv - 1);
+            if (t == 1) mma_commit(&k_empty[st ^ 1]);
+          }
+        }
+        j = jn;
+        k += boundary;
+      }
+    }
+  } else {  // ---------------------------------------- softmax: warps 2-5 tile a, 6-9 tile b
+    const int t = (warp - 2) >> 2;
+    const int q = warp & 3;
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    const uint32_t s_addr = tmem + lane_base + C::S_COL + t * C::BKV;
+    const uint32_t o_addr = tmem + lane_base + C::o_col(t);
+    uint8_t* stage = smem + C::OFF_STAGE_P + (warp - 2) * 2 * C::STAGE_BOX;
+    const int valid_last = (int)(a.nk - (int64_t)(nkv - 1) * C::BKV);  // keys of the last tile
+    int n_st = 0;  // output boxes this warp has stored
+    bool ok = true;
+    for (int item = item0, g = 0; ok && item < a.item_end; item += item_step) {
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; j < nkv; ++j, ++g) {
+        const bool ok_j = (j == nkv - 1 && valid_last < C::BKV)
+                              ? softmax_tile<D, true>(&s_full[t], &pv_done[t], &p_full[t], g, j == 0, valid_last,
+                                                      s_addr, o_addr, a.scale_log2, m_run, l_run)
+                              : softmax_tile<D, false>(&s_full[t], &pv_done[t], &p_full[t], g, j == 0, C::BKV,
+                                                       s_addr, o_addr, a.scale_log2, m_run, l_run);
+        if (!ok_j) {
+          ok = false;
+          break;
+        }
+      }
+      // ------------------------------------------------ output: O_t / l
+      // (the next PV_t, which overwrites O_t, follows this warpgroup's next
+      // p_full arrival, issued after these loads have completed)
+      if (ok) ok = mbar_wait(&pv_done[t], (g - 1) & 1);
+      tc_fence_after();
+      const int qt = item % a.nqp, h = item / a.nqp;
+      const int64_t row0 = (int64_t)qt * kBQ + t * kTileQ + q * 32;  // this warp's 32 rows
+      const float inv = 1.0f / l_run;
+      const bool wok = __all_sync(0xffffffffu, ok);
+#pragma unroll 1
+      for (int c = 0; c < D; c += 32) {
+        uint32_t o[32];
+        tmem_ld32(o_addr + c, o);
+        tmem_wait_ld();
+        if (!wok || row0 >= a.nq) continue;  // warp-uniform
+        // The warp's 32 x 32 box leaves through shared memory and one TMA
+        // store (rows past nq are clipped by the tensor map).  Two boxes
+        // alternate; the store issued two boxes ago must have read this one.
+        uint8_t* box = stage + (n_st & 1) * C::STAGE_BOX;
+        if (lane == 0 && n_st >= 2) bulk_wait_group_read<1>();
+        __syncwarp();
+        // row `lane`: 64 bytes as four 16-byte units, unit u stored at
+        // u ^ ((lane >> 1) & 3) (the 64-byte swizzle: conflict-free writes)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          uint4 w;
+          w.x = pack_bf16(__uint_as_float(o[8 * u + 0]) * inv, __uint_as_float(o[8 * u + 1]) * inv);
+          w.y = pack_bf16(__uint_as_float(o[8 * u + 2]) * inv, __uint_as_float(o[8 * u + 3]) * inv);
+          w.z = pack_bf16(__uint_as_float(o[8 * u + 4]) * inv, __uint_as_float(o[8 * u + 5]) * inv);
+          w.w = pack_bf16(__uint_as_float(o[8 * u + 6]) * inv, __uint_as_float(o[8 * u + 7]) * inv);
+          *reinterpret_cast<uint4*>(box + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) = w;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&tmO, box, a.o_col + h * D + c, (int)row0);
+          bulk_commit_group();
+        }
+        ++n_st;
+      }
+    }
+    if (lane == 0) bulk_wait_group<0>();  // output stores complete before the CTA ends
   }
   tc_fence_before();
   __syncthreads();
@@ -390,12 +643,16 @@ int num_sms_attn() {
   return n;
 }
 
+// Items with at most this many key tiles run on persistent CTAs.
+constexpr int kPersistMaxKeyTiles = 8;
+
 template <int D>
 acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
   using C = AttnCfg<D>;
   static bool attr_done = false;
   if (!attr_done) {
     ACID_CUDA(cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    ACID_CUDA(cudaFuncSetAttribute(attn_persist_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_P));
     attr_done = true;
   }
   CUtensorMap tq, tk, tv;
@@ -414,27 +671,34 @@ acid_status launch_attn_tc(const AttnArgs& x, cudaStream_t s) {
   a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
   a.nqp = (int)((x.nq + kBQ - 1) / kBQ);
   a.item_base = 0;
+  a.item_end = 0;
   a.splits = 1;
   a.part_o = nullptr;
   a.part_ml = nullptr;
   const int items = a.nqp * x.heads;
   const int nkv_all = (int)((x.nk + C::BKV - 1) / C::BKV);
-  // Items fill whole waves of CTAS_PER_SM CTAs per SM; the items of a last,
-  // partial wave are split along the key range so that they fill one wave
-  // together, and their partial results are merged.
+  // Items fill whole waves of CTAS_PER_SM CTAs per SM (or, for short key
+  // ranges, whole rounds of persistent CTAs); the items of a last, partial
+  // wave are split along the key range so that they fill one wave together,
+  // and their partial results are merged.
   const int slots = num_sms_attn() * C::CTAS_PER_SM;
   const int full = (items / slots) * slots, tail = items - full;
   int splits = tail > 0 ? std::min(std::min(kAttnPartCtas, slots) / tail, nkv_all) : 1;
   const size_t part_need = (size_t)tail * splits * kBQ * (D + 2) * sizeof(float);
   const bool split_tail = full > 0 && tail > 0 && splits >= 2 && x.part != nullptr && x.part_bytes >= part_need;
   ProfScope prof(PROF_ATTENTION, 4.0 * (double)x.nq * (double)x.nk * D * x.heads, s);
-  if (!split_tail) {
-    attn_tc_kernel<D><<<items, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
-    ACID_CHECK_LAUNCH();
-    return ACID_OK;
+  const int main_items = split_tail ? full : items;
+  if (nkv_all <= kPersistMaxKeyTiles) {
+    // output: 32-row x 32-column boxes, one per softmax warp and column chunk
+    CUtensorMap to;
+    ACID_TRY(make_tmap_bf16_box(&to, x.out, x.nq, x.ldo, x.ldo, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B));
+    a.item_end = main_items;
+    attn_persist_kernel<D><<<std::min(main_items, slots), kAttnThreads, C::SMEM_P, s>>>(tq, tk, tv, to, a);
+  } else {
+    attn_tc_kernel<D><<<main_items, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
   }
-  attn_tc_kernel<D><<<full, kAttnThreads, C::SMEM, s>>>(tq, tk, tv, a);
   ACID_CHECK_LAUNCH();
+  if (!split_tail) return ACID_OK;
   a.item_base = full;
   a.splits = splits;
   a.part_o = static_cast<float*>(x.part);

@@ -436,21 +436,27 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }  // namespace
 
 // Row-major bf16 matrix [rows, cols] with row stride ld (elements), boxes of
-// box_rows x 64 columns, 128-byte swizzle, zero fill out of bounds.
-acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+// box_rows x box_cols, the given swizzle, zero fill out of bounds.
+acid_status make_tmap_bf16_box(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                               int box_cols, int box_rows, CUtensorMapSwizzle swizzle) {
   auto fn = encode_fn();
   ACID_REQUIRE(fn != nullptr, ACID_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
   ACID_REQUIRE(aligned(base, 16) && (ld * 2) % 16 == 0, ACID_ERR_UNSUPPORTED,
                "TMA operand must be 16-byte aligned with a row stride that is a multiple of 8 elements");
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
-  cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1u, 1u};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   ACID_REQUIRE(r == CUDA_SUCCESS, ACID_ERR_CUDA, "cuTensorMapEncodeTiled failed (code " + std::to_string((int)r) + ")");
   return ACID_OK;
+}
+
+// Boxes of box_rows x 64 columns with 128-byte swizzle (the MMA operand layout).
+acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+  return make_tmap_bf16_box(map, base, rows, cols, ld, 64, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 namespace {
