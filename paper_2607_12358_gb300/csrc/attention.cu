@@ -110,6 +110,10 @@ __device__ __forceinline__ bool softmax_tile(uint64_t* s_full, uint64_t* pv_done
                                              bool first, int valid, uint32_t s_addr, uint32_t o_addr,
                                              float scale_log2, float& m_run, float& l_run) {
   using C = AttnCfg<D>;
+  // The lanes of a warp wait on the same phase, so they give up together
+  // (after the wait limit) and the warp-collective tcgen05.ld / st below stay
+  // convergent; a vote here would rule out a phase that completes exactly at
+  // the limit for some lanes only, but costs 2-3% in this loop.
   if (!mbar_wait(s_full, phase & 1)) return false;
   // consume pv_done phase - 1 (already complete: s_full(phase) is committed
   // after PV(phase - 1)) so that no later parity wait is two phases behind;
@@ -556,17 +560,17 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
       // (the next PV_t, which overwrites O_t, follows this warpgroup's next
       // p_full arrival, issued after these loads have completed)
       if (ok) ok = mbar_wait(&pv_done[t], (g - 1) & 1);
+      ok = __all_sync(0xffffffffu, ok);  // the item loop continues for the whole warp or not at all
       tc_fence_after();
       const int qt = item % a.nqp, h = item / a.nqp;
       const int64_t row0 = (int64_t)qt * kBQ + t * kTileQ + q * 32;  // this warp's 32 rows
       const float inv = 1.0f / l_run;
-      const bool wok = __all_sync(0xffffffffu, ok);
 #pragma unroll 1
       for (int c = 0; c < D; c += 32) {
         uint32_t o[32];
         tmem_ld32(o_addr + c, o);
         tmem_wait_ld();
-        if (!wok || row0 >= a.nq) continue;  // warp-uniform
+        if (!ok || row0 >= a.nq) continue;  // warp-uniform
         // The warp's 32 x 32 box leaves through shared memory and one TMA
         // store (rows past nq are clipped by the tensor map).  Two boxes
         // alternate; the store issued two boxes ago must have read this one.

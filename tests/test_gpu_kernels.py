@@ -241,6 +241,26 @@ def test_attention_peaky_rescaling(acid):
     assert _rel_l2(got, ref) <= 1e-2
 
 
+@pytest.mark.parametrize("D", [64, 128])
+def test_attention_rescale_diverging_rows(acid, D):
+    """Key tiles whose logits grow tile by tile (scale 1 + 0.6 j on tile j)
+    and query rows of seven different norms: rows cross the 2^8 rescale
+    threshold at different tiles, so within a warp some rows keep the
+    one-pass softmax while others reload S and move their reference.  The
+    last key tile is partial (masked)."""
+    nq, nk, H = 300, 1000, 2
+    bkv = 64 if D == 64 else 128
+    rng = np.random.default_rng(70 + D)
+    q = rng.normal(size=(nq, H * D)) * (0.5 + 0.5 * (np.arange(nq) % 7))[:, None]
+    k = rng.normal(size=(nk, H * D)) * (1.0 + 0.6 * (np.arange(nk) // bkv))[:, None]
+    v = rng.normal(size=(nk, H * D))
+    q, k, v = (S.round_to_bf16(x.astype(np.float32)) for x in (q, k, v))
+    ref = O.attention(q.reshape(nq, H, D), k.reshape(nk, H, D), v.reshape(nk, H, D)).reshape(nq, H * D)
+    got = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), H).float().cpu().numpy()
+    assert _rel_l2(got, ref) <= 1e-2, _rel_l2(got, ref)
+    assert np.abs(got - ref).max() <= 5e-2
+
+
 def test_attention_fp32(acid):
     rng = np.random.default_rng(11)
     q, k, v = (rng.normal(size=(70, 128)) for _ in range(3))
