@@ -38,12 +38,12 @@ WORKLOAD = ("Wan-2.1-1.3B-shaped 480p step: 30 blocks, d=1536, 12 heads x 128, F
 CPU_SAMPLE_ROWS = 4096
 REF_SAMPLE_ROWS = 2048
 
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one ncu capture of
-# a self- and a cross-attention call at this shape, each call = the main
-# launch, the split tail launch and the merge) per attention call of the step's
-# 1:1 self/cross mix.  Valid only for the kernel source it was measured on; any
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, ncu captures of
+# a self-attention call (main launch, split tail launch and merge) and a
+# cross-attention call (one persistent launch) at this shape, each the mean of
+# two calls) per attention call of the step's 1:1 self/cross mix.  Valid only for the kernel source it was measured on; any
 # other source reports null.
-ATTN_TRAFFIC = {"source_sha256_16": "bcf60336260af114", "bytes_per_launch": (434.43e6 + 165.68e6) / 2}
+ATTN_TRAFFIC = {"source_sha256_16": "e05bde0156ae53e5", "bytes_per_launch": (436.87e6 + 159.21e6) / 2}
 
 
 def _attn_traffic():
@@ -343,7 +343,7 @@ def run_ours(args) -> None:
         "config": {"workload": WORKLOAD, "global_batch": 1, "seq_len": cfg.n_video, "parallelism": "replicas",
                    "schedule": "every step computed (tau_low = tau_high = -1); drift and decision still run",
                    "l2": "no flush: per-step working set (2.8 GB weights, >0.5 GB activations) exceeds the 129 MB L2"},
-        "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel<128> (self + cross attention)",
+        "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel<128> (self) + attn_persist_kernel<128> (cross attention)",
                      "achieved": att_tflops, "peak": peak, "unit": "TFLOP/s", "frac": att_tflops / peak,
                      "peak_source": f"bf16_tflops_sustained, {src}", "traffic": _attn_traffic(),
                      "frac_of_burst_peak": att_tflops / peaks["bf16_tflops"],

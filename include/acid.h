@@ -188,9 +188,12 @@ acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t lda, int64
  * returns ACID_OK without a launch (q and out may then be NULL).  bf16 runs on
  * tcgen05 with head_dim 64 or 128; fp32 with head_dim a multiple of 32, <= 128.
  *   workspace  optional (NULL, 0): device scratch of
- *              acid_attention_workspace_size bytes.  With it, the work that
- *              would run as a last, partly filled wave of CTAs is split along
- *              the key range and merged (same result up to summation order). */
+ *              acid_attention_workspace_size bytes.  With it, and a key range
+ *              of more than 8 key tiles (1024 keys at head_dim 128, 512 at
+ *              64), the work that would run as a last, partly filled wave of
+ *              CTAs is split along the key range and merged (same result up
+ *              to summation order).  Shorter key ranges run on persistent
+ *              CTAs and do not use it. */
 acid_status acid_attention_forward(int32_t dtype, const void* q, int64_t ldq, const void* k,
                                    int64_t ldk, const void* v, int64_t ldv, void* out, int64_t ldo,
                                    int64_t nq, int64_t nk, int32_t heads, int32_t head_dim,

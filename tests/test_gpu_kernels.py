@@ -208,8 +208,8 @@ def test_attention_persistent_items(acid, nq, nk, H, D):
     differs per head (logit spreads from about 1 to about 8), so a running max
     or sum carried from one item into the next would show; with nk = 100
     every step is an item boundary and the only key tile is masked.  Every
-    row is checked against the oracle, with and without the split last
-    round."""
+    row is checked against the oracle, with and without a workspace (short
+    key ranges leave it unused)."""
     rng = np.random.default_rng(nq + nk + H)
     scale = np.repeat(1.0 + 7.0 * (np.arange(H) % 3 == 0), D)[None, :]
     q = S.round_to_bf16((scale * rng.normal(size=(nq, H * D))).astype(np.float32))
