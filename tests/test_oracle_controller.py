@@ -179,6 +179,25 @@ def test_loop_huge_threshold_reuses_first_residual(toy):
     np.testing.assert_allclose(r.latent, x, rtol=0, atol=1e-12)
 
 
+def test_force_last_computes_the_final_step(toy):
+    """force_last overrides a skip on the final step only: with every other
+    non-warmup step reused, the last step runs the block stack (and is marked
+    forced), which the replay below does by hand."""
+    cfg, w, lat = toy
+    r = O.denoise_loop(cfg, w, lat, None, tau_low=1e9, tau_high=1e9, force_last=True)
+    assert r.computed == [True] + [False] * (cfg.steps - 2) + [True]
+    assert r.records[-1].forced and not any(rec.forced for rec in r.records[:-1])
+    sig = O.sigmas(cfg.steps)
+    x = lat.astype(np.float64)
+    si = O.step_inputs(cfg, w, x, 1000.0 * sig[0])
+    R0 = O.block_stack(cfg, w, si.h_in, si.mods, None) - si.h_in
+    for i in range(cfg.steps):
+        si = O.step_inputs(cfg, w, x, 1000.0 * sig[i])
+        h = O.block_stack(cfg, w, si.h_in, si.mods, None) if i == cfg.steps - 1 else si.h_in + R0
+        x = x + (sig[i + 1] - sig[i]) * O.final_layer(cfg, w, h, si.final_mod)
+    np.testing.assert_allclose(r.latent, x, rtol=0, atol=1e-12)
+
+
 def test_loop_signals_are_consecutive_temni_drifts(toy):
     cfg, w, lat = toy
     r = O.denoise_loop(cfg, w, lat, None)
@@ -204,6 +223,25 @@ def test_easycache_affine_model_is_exact():
     np.testing.assert_allclose(O.easycache_reuse(x_t, x_c, x_c + c), x_t + c, atol=1e-15)
     s = O.easycache_signal(2.0, x_t, x_c, x_c + c)
     assert s == pytest.approx(2.0 * np.abs(x_t - x_c).mean() / np.abs(x_c + c).mean())
+
+
+def test_easycache_rate_of_a_steeper_affine_model():
+    """A model whose output moves three times as far as its input, v = 3 x +
+    c: the transformation rate is 3 (output change over input change), the
+    drift estimate is 3 mean|x_t - x_{t-1}| / mean|v_{t-1}|, and a rate read
+    the other way round (1/3) or with the roles of input and output swapped
+    fails here."""
+    rng = np.random.default_rng(5)
+    c = rng.normal(size=(4, 6))
+    x_prev = rng.normal(size=(4, 6))
+    x_c = x_prev + 0.25 * rng.normal(size=(4, 6))
+    k = O.easycache_rate(x_c, x_prev, 3.0 * x_c + c, 3.0 * x_prev + c)
+    assert k == pytest.approx(3.0, rel=1e-14)
+    # the same step seen backwards has the same rate
+    assert O.easycache_rate(x_prev, x_c, 3.0 * x_prev + c, 3.0 * x_c + c) == pytest.approx(3.0, rel=1e-14)
+    x_t = x_c + 0.5  # every element moves by 0.5: mean|x_t - x_c| = 0.5
+    v_c = 3.0 * x_c + c
+    assert O.easycache_signal(k, x_t, x_c, v_c) == pytest.approx(1.5 / np.abs(v_c).mean(), rel=1e-14)
 
 
 def test_easycache_loop_runs_and_warms_up_two_steps():

@@ -381,6 +381,25 @@ def test_hv_single_reduces_to_attention_half_of_wan_block():
                                O.wan_block(x, m6, ww, cfg.grid, cfg.heads), atol=1e-12)
 
 
+def test_hv_single_reduces_to_ffn_half_of_wan_block():
+    """W2 = [0 | W_ff2] and no text: the single-stream block is the Wan block's
+    feed-forward branch (its attention branch gated off), with W_mlp as the
+    first FFN layer and the same shift, scale and gate."""
+    cfg = _small("wan", n_text=0, dtype="fp32")
+    ww = S.block_weights(cfg, 0, 0, block_type="wan")
+    ws = S.block_weights(cfg, 0, 0, block_type="hv_single")
+    ws["mlp"] = ww["ff1"]
+    w2 = np.zeros_like(ws["w2"][0])
+    w2[:, cfg.d:] = ww["ff2"][0]
+    ws["w2"] = (w2, ww["ff2"][1])
+    rng = np.random.default_rng(21)
+    m3 = rng.normal(size=3 * cfg.d) * 0.3
+    m6 = np.concatenate([np.zeros(3 * cfg.d), m3])
+    x = S.hidden(cfg, cfg.n_video)
+    np.testing.assert_allclose(O.hv_single_block(x, m3, ws, cfg.grid, cfg.heads, 0),
+                               O.wan_block(x, m6, ww, cfg.grid, cfg.heads), atol=1e-12)
+
+
 def test_joint_block_token_permutation_without_rope():
     """Without RoPE, joint attention has no notion of order: permuting the
     video tokens permutes the output."""
