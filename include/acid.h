@@ -260,6 +260,12 @@ typedef struct {
 typedef struct {
   const float* temb;   /* device fp32 [d]: timestep embedding after the time MLP */
   const void* ctx;     /* WAN with n_text > 0: device [n_text, d] text context, desc dtype */
+  const void* ctx_kv;  /* optional (NULL): WAN with n_text > 0: device [n_text, 2d], desc dtype,
+                          16-byte aligned, this block's cross-attention keys and values
+                          ctx W_ckv^T + b_ckv (keys in columns [0, d), values in [d, 2d)).
+                          The text is fixed for a generation, so a caller running many
+                          steps computes them once per block (acid_denoise_* do); given,
+                          the block reads them and ctx may be NULL. */
 } acid_cond;
 
 /* Rows of x for a block: n_video (WAN) or n_text + n_video (COG/HV). */

@@ -39,7 +39,7 @@ class acid_block_weights(C.Structure):
 
 
 class acid_cond(C.Structure):
-    _fields_ = [("temb", C.c_void_p), ("ctx", C.c_void_p)]
+    _fields_ = [("temb", C.c_void_p), ("ctx", C.c_void_p), ("ctx_kv", C.c_void_p)]
 
 
 class acid_model(C.Structure):

@@ -247,14 +247,17 @@ class DeviceBlock:
 
 def acid_dit_block_forward(desc: A.acid_block_desc, x: torch.Tensor, temb: torch.Tensor,
                            block: DeviceBlock, ctx: torch.Tensor | None = None,
-                           workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
-    """One block in place on x [rows, d]; temb fp32 [d]; ctx [n_text, d] (WAN)."""
-    _need_cuda(x, temb, ctx)
+                           workspace: torch.Tensor | None = None, stream=None,
+                           ctx_kv: torch.Tensor | None = None) -> torch.Tensor:
+    """One block in place on x [rows, d]; temb fp32 [d]; ctx [n_text, d] (WAN);
+    ctx_kv [n_text, 2d] (WAN, optional): the block's cross-attention keys and
+    values computed ahead, used instead of projecting ctx."""
+    _need_cuda(x, temb, ctx, ctx_kv)
     if workspace is None:
         workspace = torch.empty(block_workspace_size(desc) + 1024, dtype=torch.uint8, device=x.device)
     base = workspace.data_ptr()
     aligned = (base + 1023) // 1024 * 1024
-    cond = A.acid_cond(temb.data_ptr(), _ptr(ctx))
+    cond = A.acid_cond(temb.data_ptr(), _ptr(ctx), _ptr(ctx_kv))
     check(load().acid_dit_block_forward(C.byref(desc), x.data_ptr(), C.byref(cond), C.byref(block.struct),
                                         aligned, workspace.numel() - (aligned - base), _stream(stream)))
     return x

@@ -103,8 +103,8 @@ acid_status validate_block_weights(const acid_block_desc& d, const acid_block_we
 }
 
 acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* temb, const void* ctx,
-                               const acid_block_weights& W, const BlockWs& ws, const RopeTable* rope_in,
-                               cudaStream_t s) {
+                               const void* ctx_kv, const acid_block_weights& W, const BlockWs& ws,
+                               const RopeTable* rope_in, cudaStream_t s) {
   const int dt = D.dtype;
   const int d = D.d, F = D.ffn, hd = d / D.heads;
   const int64_t L = D.kind == ACID_BLOCK_WAN ? 0 : D.n_text;  // joint text rows
@@ -225,11 +225,14 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
     ACID_TRY(ln_mod(ACID_FP32, xm, dt, ws.u, rows, d, nullptr, nullptr, nullptr, nullptr, 0, eps, s));
     Epilogue eb;
     ACID_TRY(lin(dt, ws.u, d, rows, d, W.cq, d, ws.att, d, eb, s));
-    ACID_TRY(lin(dt, ctx, d, D.n_text, d, W.ckv, 2 * d, ws.kvc, 2 * d, eb, s));
+    if (ctx_kv == nullptr) {
+      ACID_TRY(lin(dt, ctx, d, D.n_text, d, W.ckv, 2 * d, ws.kvc, 2 * d, eb, s));
+      ctx_kv = ws.kvc;
+    }
     AttnArgs cross;
     cross.q = ws.att;
     cross.ldq = d;
-    cross.k = cross.v = ws.kvc;
+    cross.k = cross.v = ctx_kv;
     cross.ldk = cross.ldv = 2 * (int64_t)d;
     cross.k_col = 0;
     cross.v_col = d;
@@ -295,13 +298,15 @@ extern "C" acid_status acid_dit_block_forward(const acid_block_desc* desc, void*
   ACID_TRY(validate_block_desc(*desc));
   ACID_TRY(validate_block_weights(*desc, *w));
   ACID_REQUIRE(cond->temb != nullptr, ACID_ERR_INVALID_ARG, "acid_dit_block_forward: cond->temb is null");
-  ACID_REQUIRE(!(desc->kind == ACID_BLOCK_WAN && desc->n_text > 0) || cond->ctx != nullptr, ACID_ERR_INVALID_ARG,
-               "acid_dit_block_forward: WAN cross-attention needs cond->ctx");
+  ACID_REQUIRE(!(desc->kind == ACID_BLOCK_WAN && desc->n_text > 0) || cond->ctx != nullptr || cond->ctx_kv != nullptr,
+               ACID_ERR_INVALID_ARG, "acid_dit_block_forward: WAN cross-attention needs cond->ctx or cond->ctx_kv");
+  ACID_REQUIRE(cond->ctx_kv == nullptr || aligned(cond->ctx_kv, 16), ACID_ERR_UNSUPPORTED,
+               "acid_dit_block_forward: cond->ctx_kv must be 16-byte aligned");
   ACID_REQUIRE(aligned(x, 16), ACID_ERR_UNSUPPORTED, "acid_dit_block_forward: x must be 16-byte aligned");
   ACID_REQUIRE(workspace != nullptr && aligned(workspace, 1024), ACID_ERR_WORKSPACE,
                "acid_dit_block_forward: workspace must be non-null and 1024-byte aligned");
   BlockWs ws = block_ws_layout(*desc, workspace);
   ACID_REQUIRE(workspace_bytes >= ws.bytes, ACID_ERR_WORKSPACE,
                "acid_dit_block_forward: workspace too small (need " + std::to_string(ws.bytes) + " bytes)");
-  return block_forward_impl(*desc, x, cond->temb, cond->ctx, *w, ws, nullptr, (cudaStream_t)stream);
+  return block_forward_impl(*desc, x, cond->temb, cond->ctx, cond->ctx_kv, *w, ws, nullptr, (cudaStream_t)stream);
 }

@@ -41,8 +41,10 @@ int64_t block_rows(const acid_block_desc& d);
 BlockWs block_ws_layout(const acid_block_desc& d, void* base);
 acid_status validate_block_desc(const acid_block_desc& d);
 acid_status validate_block_weights(const acid_block_desc& d, const acid_block_weights& w);
+// ctx_kv: this block's cross-attention keys and values [n_text, 2d] computed
+// ahead (the text is fixed for a generation), or null to project ctx here.
 acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* temb, const void* ctx,
-                               const acid_block_weights& W, const BlockWs& ws, const RopeTable* rope,
-                               cudaStream_t s);
+                               const void* ctx_kv, const acid_block_weights& W, const BlockWs& ws,
+                               const RopeTable* rope, cudaStream_t s);
 
 }  // namespace acid

@@ -34,6 +34,7 @@ struct LoopWs {
   float* resid;     // [N, d] TeaCache residual H_out - H_in
   uint8_t* xbuf;    // [L + N, d] block-stack state (model dtype)
   uint8_t* text;    // [L, d] text context / text tokens (model dtype)
+  uint8_t* ctx_kv;  // WAN with text: [blocks, L, 2d] cross-attention keys and values (model dtype)
   uint8_t* y;       // [N, d] final LayerNorm output
   float* vtok;      // [N, P] final layer output
   float* v[2];      // latent-sized velocity, current / previous (EasyCache)
@@ -119,6 +120,8 @@ LoopWs loop_layout(const acid_model& m, void* base) {
   const int64_t xrows = m.block.kind == ACID_BLOCK_WAN ? s.N : s.N + s.L;
   w.xbuf = b.take<uint8_t>(xrows * s.d * es(dt));
   w.text = b.take<uint8_t>(std::max<int64_t>(s.L, 1) * s.d * es(dt));
+  const bool wan_text = m.block.kind == ACID_BLOCK_WAN && s.L > 0;
+  w.ctx_kv = b.take<uint8_t>(wan_text ? (size_t)total_blocks(m) * s.L * 2 * s.d * es(dt) : 0);
   w.y = b.take<uint8_t>(s.N * s.d * es(dt));
   w.vtok = b.take<float>(s.N * s.P);
   w.v[0] = b.take<float>(s.latent);
@@ -265,12 +268,15 @@ acid_status run_blocks(const acid_model& m, const LoopWs& w, cudaStream_t s, int
     t.table = w.rope;
     return t;
   }();
-  const void* ctx = m.block.kind == ACID_BLOCK_WAN && m.block.n_text > 0 ? w.text : nullptr;
+  const bool wan_text = m.block.kind == ACID_BLOCK_WAN && m.block.n_text > 0;
+  const void* ctx = wan_text ? w.text : nullptr;
+  const size_t kv_bytes = (size_t)m.block.n_text * 2 * m.block.d * es(m.block.dtype);
   if (b1 < 0) b1 = total_blocks(m);
   for (int i = b0; i < b1; ++i) {
     const acid_block_desc d = desc_for(m, i);
     const BlockWs bws = block_ws_layout(d, w.block_base);
-    ACID_TRY(block_forward_impl(d, w.xbuf, w.temb, ctx, m.blocks[i], bws, &base_rope, s));
+    const void* kv = wan_text ? w.ctx_kv + i * kv_bytes : nullptr;
+    ACID_TRY(block_forward_impl(d, w.xbuf, w.temb, ctx, kv, m.blocks[i], bws, &base_rope, s));
   }
   return ACID_OK;
 }
@@ -403,6 +409,15 @@ extern "C" acid_status acid_loop_begin(const acid_model* m, const acid_loop_cfg*
       Epilogue e;
       e.bias = m->text.b;
       ACID_TRY(linear_forward(dt, text, m->d_text, sh.L, m->d_text, m->text.w, sh.d, w.text, sh.d, e, s));
+      // every block's cross-attention keys and values, once per generation
+      // (the same GEMM the block would run on each step)
+      const size_t kv_bytes = (size_t)sh.L * 2 * sh.d * es(dt);
+      for (int i = 0; i < total_blocks(*m); ++i) {
+        Epilogue ekv;
+        ekv.bias = m->blocks[i].ckv.b;
+        ACID_TRY(linear_forward(dt, w.text, sh.d, sh.L, sh.d, m->blocks[i].ckv.w, 2 * sh.d, w.ctx_kv + i * kv_bytes,
+                                2 * sh.d, ekv, s));
+      }
     } else {
       ACID_CUDA(cudaMemcpyAsync(w.text, text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
     }

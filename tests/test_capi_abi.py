@@ -60,7 +60,7 @@ _PROBE = r"""
 int main(void) {
   P(acid_block_desc) O(acid_block_desc, n_text) O(acid_block_desc, ln_eps)
   P(acid_linear) P(acid_block_weights) O(acid_block_weights, t_ff2)
-  P(acid_cond) P(acid_model) O(acid_model, blocks) O(acid_model, d_text) O(acid_model, final_out)
+  P(acid_cond) O(acid_cond, ctx_kv) P(acid_model) O(acid_model, blocks) O(acid_model, d_text) O(acid_model, final_out)
   P(acid_loop_cfg) O(acid_loop_cfg, tau_low) O(acid_loop_cfg, forced) O(acid_loop_cfg, probe_blocks) O(acid_loop_cfg, signal_poly)
   O(acid_loop_cfg, tau_schedule)
   P(acid_step_log) O(acid_step_log, ms) P(acid_loop_state) O(acid_loop_state, k_rate)

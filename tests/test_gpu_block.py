@@ -78,6 +78,29 @@ def test_wan_block_bf16(acid, heads, d, q_scale):
     _check(got, ref, x, True)
 
 
+def test_wan_block_cross_kv_computed_ahead_is_identical(acid):
+    """The cross-attention keys and values computed ahead (the step loop does
+    it once per generation: the text is fixed) give the block output of the
+    block that projects the text itself, bit for bit, and the oracle's."""
+    cfg = S.get_config("wan", d=256, heads=2, ffn=512, n_text=77, **SMALL)
+    w = S.block_weights(cfg, 0, seed=3)
+    x = S.hidden(cfg, cfg.n_video, seed=3)
+    temb = S.temb_vector(cfg, seed=3)
+    ctx = S.round_to_bf16(S.normal(3, (cfg.n_text, cfg.d), 1.0, "ctx"))
+    blk = acid.DeviceBlock.upload(w, "wan", torch.bfloat16, DEV)
+    desc = acid.block_desc(cfg, "wan")
+    t_temb, t_ctx = _t(temb, torch.float32), _t(ctx, torch.bfloat16)
+    a = acid.acid_dit_block_forward(desc, _t(x, torch.bfloat16), t_temb, blk, ctx=t_ctx)
+    kw, kb = blk.tensors["ckv"]
+    kv = acid.acid_linear_forward(t_ctx, kw, kb)
+    b = acid.acid_dit_block_forward(desc, _t(x, torch.bfloat16), t_temb, blk, ctx=None, ctx_kv=kv)
+    torch.cuda.synchronize()
+    acid.check_device_error()
+    assert torch.equal(a, b)
+    ref = O.wan_block(x, O.block_modulation(temb, w["mod"]), w, cfg.grid, cfg.heads, ctx=ctx)
+    _check(b.float().cpu().numpy(), ref, x, True)
+
+
 def test_toy_block_fp32(acid):
     cfg = S.get_config("toy")
     w = S.block_weights(cfg, 0, seed=2, q_scale=4.0)
