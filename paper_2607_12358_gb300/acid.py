@@ -165,7 +165,8 @@ def acid_attention_forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, he
                            out: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
                            stream=None) -> torch.Tensor:
     """softmax(q k^T / sqrt(Dh)) v per head; q [nq, H*Dh], k/v [nk, H*Dh] (row strides taken from the tensors).
-    ``workspace`` (optional, attention_workspace_size bytes) enables the split of a partial last wave."""
+    ``workspace`` (optional, attention_workspace_size bytes) enables the split of a partial last wave for key
+    ranges of more than 8 key tiles; shorter ones run on persistent CTAs and leave it unused."""
     _need_cuda(q, k, v, out, workspace)
     nq, nk = q.shape[0], k.shape[0]
     hd = q.shape[1] // heads
