@@ -199,6 +199,41 @@ __device__ __forceinline__ bool softmax_tile(uint64_t* s_full, uint64_t* pv_done
   return true;
 }
 
+// S_t = Q_t K^T for one key tile: D/16 MMAs (M128, N = BKV, K16) into TMEM
+// column d; qdesc_t / kdesc_slot: shared-memory descriptors of Q_t and of the
+// K ring slot (an operand at byte offset o is the descriptor plus o >> 4).
+template <int D>
+__device__ __forceinline__ void issue_s_mma(uint32_t d, uint64_t qdesc_t, uint64_t kdesc_slot) {
+  using C = AttnCfg<D>;
+  constexpr uint32_t idesc_s = idesc_bf16_f32(128, C::BKV, false, false);
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const uint64_t off_a = (uint64_t)(((kk >> 2) * C::CHUNK_Q + (kk & 3) * 32) >> 4);
+    const uint64_t off_b = (uint64_t)(((kk >> 2) * C::CHUNK_KV + (kk & 3) * 32) >> 4);
+    mma_bf16_ss(d, qdesc_t + off_a, kdesc_slot + off_b, idesc_s, kk != 0);
+  }
+}
+
+// O_t (+)= P_t V for one key tile: BKV/16 MMAs (M128, N = D, K16), P_t from
+// TMEM at column p (bf16 pairs over the S region), V MN-major from the ring
+// slot; accumulate is false on an item's first key tile.
+template <int D>
+__device__ __forceinline__ void issue_pv_mma(uint32_t d, uint32_t p, uint64_t vdesc_slot, bool accumulate) {
+  using C = AttnCfg<D>;
+  constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
+#pragma unroll
+  for (int kk = 0; kk < C::BKV / 16; ++kk)
+    mma_bf16_ts(d, p + kk * 8, vdesc_slot + (uint64_t)((kk * 16 * 128) >> 4), idesc_o, accumulate || kk != 0);
+}
+
+// TMA loads of one K or V tile (D / 64 chunks of 64 columns) into a ring slot.
+template <int D>
+__device__ __forceinline__ void load_kv_tile(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int col, int row) {
+  using C = AttnCfg<D>;
+  mbar_expect_tx(bar, C::KV_BYTES);
+  for (int c = 0; c < C::CH; ++c) tma_load_2d(dst + c * C::CHUNK_KV, map, bar, col + c * 64, row);
+}
+
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -259,21 +294,13 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
       for (int j = 0; j < nkv; ++j) {
         const int st = j & 1, round = j >> 1;
         if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) break;
-        mbar_expect_tx(&k_full[st], C::KV_BYTES);
-        for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sK + st * C::KV_BYTES + c * C::CHUNK_KV, &tmK, &k_full[st], a.k_col + h * D + c * 64,
-                      (jb + j) * C::BKV);
+        load_kv_tile<D>(sK + st * C::KV_BYTES, &tmK, &k_full[st], a.k_col + h * D, (jb + j) * C::BKV);
         if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) break;
-        mbar_expect_tx(&v_full[st], C::KV_BYTES);
-        for (int c = 0; c < C::CH; ++c)
-          tma_load_2d(sV + st * C::KV_BYTES + c * C::CHUNK_KV, &tmV, &v_full[st], a.v_col + h * D + c * 64,
-                      (jb + j) * C::BKV);
+        load_kv_tile<D>(sV + st * C::KV_BYTES, &tmV, &v_full[st], a.v_col + h * D, (jb + j) * C::BKV);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------------------------------- MMA issuer
-      constexpr uint32_t idesc_s = idesc_bf16_f32(128, C::BKV, false, false);
-      constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
       // Shared-memory descriptors are built once; an operand at byte offset o
       // from a base is the base descriptor plus o >> 4 (the 14-bit address
       // field cannot overflow: shared memory ends below 256 KB).
@@ -282,15 +309,8 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
       const uint64_t vdesc = smem_desc_sw128(smem_u32(sV), C::CHUNK_KV, 1024);
       // S_t(j) = Q_t K_j^T into the S region of tile t
       auto issue_s = [&](int t, int j) {
-        const uint64_t a0 = qdesc + (uint64_t)((t * C::T_BYTES) >> 4);
-        const uint64_t b0 = kdesc + (uint64_t)(((j & 1) * C::KV_BYTES) >> 4);
-        const uint32_t d = tmem + C::S_COL + t * C::BKV;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t off_a = (uint64_t)(((kk >> 2) * C::CHUNK_Q + (kk & 3) * 32) >> 4);
-          const uint64_t off_b = (uint64_t)(((kk >> 2) * C::CHUNK_KV + (kk & 3) * 32) >> 4);
-          mma_bf16_ss(d, a0 + off_a, b0 + off_b, idesc_s, kk != 0);
-        }
+        issue_s_mma<D>(tmem + C::S_COL + t * C::BKV, qdesc + (uint64_t)((t * C::T_BYTES) >> 4),
+                       kdesc + (uint64_t)(((j & 1) * C::KV_BYTES) >> 4));
         mma_commit(&s_full[t]);
       };
       bool ok = mbar_wait(q_full, 0) && mbar_wait(&k_full[0], 0);
@@ -306,12 +326,9 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
           if (!mbar_wait(&p_full[t], j & 1)) { ok = false; break; }
           if (t == 0 && !mbar_wait(&v_full[st], (j >> 1) & 1)) { ok = false; break; }
           tc_fence_after();
-          // O_t += P_t V_j: P_t (128 x 128 keys) from TMEM, V_j MN-major from shared memory
-          const uint64_t b0 = vdesc + (uint64_t)((st * C::KV_BYTES) >> 4);
-          const uint32_t d = tmem + C::o_col(t), p0 = tmem + C::S_COL + t * C::BKV;
-#pragma unroll
-          for (int kk = 0; kk < C::BKV / 16; ++kk)
-            mma_bf16_ts(d, p0 + kk * 8, b0 + (uint64_t)((kk * 16 * 128) >> 4), idesc_o, (j | kk) != 0);
+          // O_t += P_t V_j
+          issue_pv_mma<D>(tmem + C::o_col(t), tmem + C::S_COL + t * C::BKV,
+                          vdesc + (uint64_t)((st * C::KV_BYTES) >> 4), j != 0);
           mma_commit(&pv_done[t]);
           if (t == 1) mma_commit(&v_empty[st]);
           if (j + 1 < nkv) {
@@ -463,37 +480,22 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
         for (int j = 0; ok && j < nkv; ++j, ++g) {
           const int st = g & 1, round = g >> 1;
           if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) { ok = false; break; }
-          mbar_expect_tx(&k_full[st], C::KV_BYTES);
-          for (int c = 0; c < C::CH; ++c)
-            tma_load_2d(sK + st * C::KV_BYTES + c * C::CHUNK_KV, &tmK, &k_full[st], a.k_col + h * D + c * 64,
-                        j * C::BKV);
+          load_kv_tile<D>(sK + st * C::KV_BYTES, &tmK, &k_full[st], a.k_col + h * D, j * C::BKV);
           if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) { ok = false; break; }
-          mbar_expect_tx(&v_full[st], C::KV_BYTES);
-          for (int c = 0; c < C::CH; ++c)
-            tma_load_2d(sV + st * C::KV_BYTES + c * C::CHUNK_KV, &tmV, &v_full[st], a.v_col + h * D + c * 64,
-                        j * C::BKV);
+          load_kv_tile<D>(sV + st * C::KV_BYTES, &tmV, &v_full[st], a.v_col + h * D, j * C::BKV);
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------------------------------- MMA issuer
-      constexpr uint32_t idesc_s = idesc_bf16_f32(128, C::BKV, false, false);
-      constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
       const uint64_t qdesc = smem_desc_sw128(smem_u32(sQ), 16, 1024);
       const uint64_t kdesc = smem_desc_sw128(smem_u32(sK), 16, 1024);
       const uint64_t vdesc = smem_desc_sw128(smem_u32(sV), C::CHUNK_KV, 1024);
       // S_t = Q_t K^T of step g into the S region of tile t; after an item's
       // last key tile (last_tile) the producer may replace Q_t
       auto issue_s = [&](int t, int g, bool last_tile) {
-        const uint64_t a0 = qdesc + (uint64_t)((t * C::T_BYTES) >> 4);
-        const uint64_t b0 = kdesc + (uint64_t)(((g & 1) * C::KV_BYTES) >> 4);
-        const uint32_t d = tmem + C::S_COL + t * C::BKV;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t off_a = (uint64_t)(((kk >> 2) * C::CHUNK_Q + (kk & 3) * 32) >> 4);
-          const uint64_t off_b = (uint64_t)(((kk >> 2) * C::CHUNK_KV + (kk & 3) * 32) >> 4);
-          mma_bf16_ss(d, a0 + off_a, b0 + off_b, idesc_s, kk != 0);
-        }
+        issue_s_mma<D>(tmem + C::S_COL + t * C::BKV, qdesc + (uint64_t)((t * C::T_BYTES) >> 4),
+                       kdesc + (uint64_t)(((g & 1) * C::KV_BYTES) >> 4));
         mma_commit(&s_full[t]);
         if (last_tile) mma_commit(&q_empty[t]);
       };
@@ -514,11 +516,8 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
           if (!mbar_wait(&p_full[t], g & 1)) { ok = false; break; }
           if (t == 0 && !mbar_wait(&v_full[st], (g >> 1) & 1)) { ok = false; break; }
           tc_fence_after();
-          const uint64_t b0 = vdesc + (uint64_t)((st * C::KV_BYTES) >> 4);
-          const uint32_t d = tmem + C::o_col(t), p0 = tmem + C::S_COL + t * C::BKV;
-#pragma unroll
-          for (int kk = 0; kk < C::BKV / 16; ++kk)
-            mma_bf16_ts(d, p0 + kk * 8, b0 + (uint64_t)((kk * 16 * 128) >> 4), idesc_o, (j | kk) != 0);
+          issue_pv_mma<D>(tmem + C::o_col(t), tmem + C::S_COL + t * C::BKV,
+                          vdesc + (uint64_t)((st * C::KV_BYTES) >> 4), j != 0);
           mma_commit(&pv_done[t]);
           if (t == 1) mma_commit(&v_empty[st]);
           if (gn < total) {
