@@ -43,7 +43,7 @@ REF_SAMPLE_ROWS = 2048
 # cross-attention call (one persistent launch) at this shape, each the mean of
 # two calls) per attention call of the step's 1:1 self/cross mix.  Valid only for the kernel source it was measured on; any
 # other source reports null.
-ATTN_TRAFFIC = {"source_sha256_16": "e05bde0156ae53e5", "bytes_per_launch": (436.87e6 + 159.21e6) / 2}
+ATTN_TRAFFIC = {"source_sha256_16": "f4686df233990ff3", "bytes_per_launch": (435.47e6 + 159.20e6) / 2}
 
 
 def _attn_traffic():
