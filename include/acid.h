@@ -174,23 +174,13 @@ typedef enum {
  *   out        device [M, N] row stride ldo; fp32 if out_fp32 else dtype.
  *   gate       fp32 [N] (ACID_EPI_GATED_RES), residual [M, N] row stride ldr
  *              in the output dtype (may equal out: in place).
- *   workspace  optional (NULL, 0): device scratch of acid_linear_workspace_size
- *              bytes, 16-byte aligned.  With it, a bf16 layer whose 128 x 256
- *              output tiles leave a partial last round on the SMs splits that
- *              round along K (at least 1024 of K per split) and adds the parts
- *              in a fixed order before the epilogue: the same result up to
- *              summation order, deterministic.
  * bf16 runs on tcgen05 (fp32 accumulation): N % 32 == 0, K % 8 == 0, rows
  * 16-byte aligned.  fp32 runs on the FP32 pipes: N even.  M = 0 returns
  * ACID_OK without a launch (the pointers may then be NULL). */
 acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t lda, int64_t M, int32_t K,
                                 const void* W, const float* bias, int32_t N, void* out, int64_t ldo,
                                 int32_t epilogue, const float* gate, const void* residual,
-                                int64_t ldr, int32_t out_fp32, void* workspace, size_t workspace_bytes,
-                                acid_stream_t stream);
-/* Bytes of the optional acid_linear_forward workspace (fp32 partial tiles
- * for up to 160 CTAs). */
-acid_status acid_linear_workspace_size(size_t* bytes);
+                                int64_t ldr, int32_t out_fp32, acid_stream_t stream);
 
 /* Multi-head attention softmax(q k^T / sqrt(head_dim)) v, per head h reading
  * columns [h*head_dim, (h+1)*head_dim) of q (row stride ldq), k (ldk), v (ldv)

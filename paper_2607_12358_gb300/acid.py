@@ -139,19 +139,11 @@ def acid_drift_apply(prev, cur, cached_residual, out=None, out_rel=None, out_sum
 _EPI = {"bias": A.ACID_EPI_BIAS, "gelu": A.ACID_EPI_GELU, "gated_res": A.ACID_EPI_GATED_RES, "res": A.ACID_EPI_RES}
 
 
-def linear_workspace_size() -> int:
-    b = C.c_size_t()
-    check(load().acid_linear_workspace_size(C.byref(b)))
-    return b.value
-
-
 def acid_linear_forward(a: torch.Tensor, w: torch.Tensor, bias: torch.Tensor | None = None, epilogue: str = "bias",
                         gate: torch.Tensor | None = None, residual: torch.Tensor | None = None,
-                        out: torch.Tensor | None = None, out_fp32: bool = False, stream=None,
-                        workspace: torch.Tensor | None = None) -> torch.Tensor:
-    """out = epilogue(a @ w.T + bias); a [M, K] (row stride a.stride(0)), w [N, K].
-    ``workspace`` (optional, linear_workspace_size bytes) lets a partial last round of tiles split along K."""
-    _need_cuda(a, w, bias, gate, residual, out, workspace)
+                        out: torch.Tensor | None = None, out_fp32: bool = False, stream=None) -> torch.Tensor:
+    """out = epilogue(a @ w.T + bias); a [M, K] (row stride a.stride(0)), w [N, K]."""
+    _need_cuda(a, w, bias, gate, residual, out)
     M, K = a.shape
     N = w.shape[0]
     if out is None:
@@ -159,9 +151,7 @@ def acid_linear_forward(a: torch.Tensor, w: torch.Tensor, bias: torch.Tensor | N
         out = torch.empty(M, N, dtype=odt, device=a.device)
     check(load().acid_linear_forward(_dtype(a), a.data_ptr(), a.stride(0), M, K, w.data_ptr(), _ptr(bias), N,
                                      out.data_ptr(), out.stride(0), _EPI[epilogue], _ptr(gate), _ptr(residual),
-                                     0 if residual is None else residual.stride(0), int(out_fp32), _ptr(workspace),
-                                     0 if workspace is None else workspace.numel() * workspace.element_size(),
-                                     _stream(stream)))
+                                     0 if residual is None else residual.stride(0), int(out_fp32), _stream(stream)))
     return out
 
 

@@ -21,8 +21,8 @@ const void* coff(const void* base, int64_t elems, int dtype) {
   return static_cast<const uint8_t*>(base) + elems * (int64_t)esize(dtype);
 }
 
-acid_status lin_w(int dt, const void* A, int64_t lda, int64_t M, int K, const acid_linear& L, int N, void* out,
-                  int64_t ldo, Epilogue e, cudaStream_t s) {
+acid_status lin(int dt, const void* A, int64_t lda, int64_t M, int K, const acid_linear& L, int N, void* out,
+                int64_t ldo, Epilogue e, cudaStream_t s) {
   e.bias = L.b;
   return linear_forward(dt, A, lda, M, K, L.w, N, out, ldo, e, s);
 }
@@ -52,8 +52,6 @@ BlockWs block_ws_layout(const acid_block_desc& d, void* base) {
   if (d.dtype == ACID_BF16 && d.heads > 0) {
     w.attn_part_bytes = attn_part_bytes(d.d / d.heads);
     w.attn_part = b.take<uint8_t>(w.attn_part_bytes);
-    w.gemm_split_bytes = kGemmSplitBytes;
-    w.gemm_split = b.take<float>(kGemmSplitBytes / sizeof(float));
   }
   w.kvc = (d.kind == ACID_BLOCK_WAN && d.n_text > 0) ? b.take<uint8_t>(d.n_text * 2 * (int64_t)d.d * es) : nullptr;
   w.bytes = b.off + 1024;
@@ -109,13 +107,6 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
                                const RopeTable* rope_in, cudaStream_t s) {
   const int dt = D.dtype;
   const int d = D.d, F = D.ffn, hd = d / D.heads;
-  // every linear layer of the block may split its partial last round of tiles
-  auto lin = [&](int dt_, const void* A, int64_t lda, int64_t M, int K, const acid_linear& L, int N, void* out,
-                 int64_t ldo, Epilogue e, cudaStream_t st) {
-    e.split_ws = ws.gemm_split;
-    e.split_ws_bytes = ws.gemm_split_bytes;
-    return lin_w(dt_, A, lda, M, K, L, N, out, ldo, e, st);
-  };
   const int64_t L = D.kind == ACID_BLOCK_WAN ? 0 : D.n_text;  // joint text rows
   const int64_t rows = block_rows(D);
   const int64_t Nv = rows - L;

@@ -34,8 +34,6 @@ struct BlockWs {
   float* xm = nullptr;     // [rows, d] fp32 residual stream between the two branches
   void* attn_part = nullptr;  // attention partial results of a split last wave
   size_t attn_part_bytes = 0;
-  float* gemm_split = nullptr;  // linear layers: partial tiles of a split last round
-  size_t gemm_split_bytes = 0;
   size_t bytes = 0;
 };
 

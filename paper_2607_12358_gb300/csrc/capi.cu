@@ -201,8 +201,7 @@ extern "C" acid_status acid_cache_apply(const void* x, const void* cached_residu
 extern "C" acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t lda, int64_t M, int32_t K,
                                            const void* W, const float* bias, int32_t N, void* out, int64_t ldo,
                                            int32_t epilogue, const float* gate, const void* residual, int64_t ldr,
-                                           int32_t out_fp32, void* workspace, size_t workspace_bytes,
-                                           acid_stream_t stream) {
+                                           int32_t out_fp32, acid_stream_t stream) {
   clear_error();
   ACID_REQUIRE(dtype == ACID_BF16 || dtype == ACID_FP32, ACID_ERR_INVALID_ARG, "acid_linear_forward: unknown dtype");
   ACID_REQUIRE(epilogue == ACID_EPI_BIAS || epilogue == ACID_EPI_GELU || epilogue == ACID_EPI_GATED_RES ||
@@ -219,18 +218,7 @@ extern "C" acid_status acid_linear_forward(int32_t dtype, const void* A, int64_t
   e.ldr = ldr;
   e.out_fp32 = out_fp32 != 0 || dtype == ACID_FP32;
   e.res_fp32 = e.out_fp32;  // the residual has the output's dtype
-  ACID_REQUIRE(workspace == nullptr || aligned(workspace, 16), ACID_ERR_WORKSPACE,
-               "acid_linear_forward: workspace must be 16-byte aligned");
-  e.split_ws = static_cast<float*>(workspace);
-  e.split_ws_bytes = workspace ? workspace_bytes : 0;
   return linear_forward(dtype, A, lda, M, K, W, N, out, ldo, e, (cudaStream_t)stream);
-}
-
-extern "C" acid_status acid_linear_workspace_size(size_t* bytes) {
-  clear_error();
-  ACID_REQUIRE(bytes != nullptr, ACID_ERR_INVALID_ARG, "acid_linear_workspace_size: null argument");
-  *bytes = kGemmSplitBytes;
-  return ACID_OK;
 }
 
 extern "C" acid_status acid_attention_forward(int32_t dtype, const void* q, int64_t ldq, const void* k, int64_t ldk,

@@ -161,11 +161,6 @@ struct GemmDims {
   void* out;
   int64_t ldo;
   int out_fp32;
-  int tile_end;    // the persistent CTAs take tiles [0, tile_end)
-  // split round: tile split_base + i runs on CTAs i * splits .. + splits - 1,
-  // each over a K range, writing fp32 partial tiles [CTA][BN/32][128][32] to part
-  int split_base, splits;
-  float* part;
 };
 
 // Epilogue of 32-row x 32-column accumulator chunks held by a warp (thread =
@@ -295,10 +290,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
   __syncwarp();
 }
 
-// SPLIT: one tile of a split round per CTA, over its K range, with the raw
-// accumulator stored to g.part (gemm_split_fixup_kernel adds the parts and
-// applies the epilogue).
-template <int BN, int KIND, bool R32, bool SPLIT = false>
+template <int BN, int KIND, bool R32>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
                    EpiDev e) {
@@ -316,16 +308,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int num_kb = (g.K + BK - 1) / BK;
   const int num_n = (g.N + BN - 1) / BN;
-  // this CTA's tiles (first, first + step, ... below last) and K blocks [kb0, kb1)
-  int tile_first = blockIdx.x, tile_last = g.tile_end, tile_step = gridDim.x, kb0 = 0, kb1 = num_kb;
-  if constexpr (SPLIT) {
-    const int sp = (int)blockIdx.x % g.splits;
-    tile_first = g.split_base + (int)blockIdx.x / g.splits;
-    tile_last = tile_first + 1;
-    tile_step = 1;
-    kb0 = (int)((int64_t)sp * num_kb / g.splits);
-    kb1 = (int)((int64_t)(sp + 1) * num_kb / g.splits);
-  }
+  const int num_tiles = (int)((g.M + BM - 1) / BM) * num_n;
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
@@ -350,9 +333,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (lane == 0) {  // TMA producer: one continuous stage ring across tiles
       int it = 0;
       bool ok = true;
-      for (int tile = tile_first; ok && tile < tile_last; tile += tile_step) {
+      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
         const int m_tile = tile / num_n, n_tile = tile % num_n;
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES, round = it / C::STAGES;
           if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1)) { ok = false; break; }
           mbar_expect_tx(&full[s], C::STAGE_BYTES);
@@ -366,12 +349,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
       int it = 0, local = 0;
       bool ok = true;
-      for (int tile = tile_first; ok && tile < tile_last; tile += tile_step, ++local) {
+      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++local) {
         const int b = local & 1, use = local >> 1;
         if (use > 0 && !mbar_wait(&acc_empty[b], (use - 1) & 1)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d = tmem + b * BN;
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES, round = it / C::STAGES;
           if (!mbar_wait(&full[s], round & 1)) { ok = false; break; }
           tc_fence_after();
@@ -381,7 +364,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = smem_desc_sw128(a0 + k * 32, 16, 1024);
             const uint64_t bd = smem_desc_sw128(b0 + k * 32, 16, 1024);
-            mma_bf16_ss(d, ad, bd, idesc, kb != kb0 || k != 0);
+            mma_bf16_ss(d, ad, bd, idesc, (kb | k) != 0);
           }
           mma_commit(&empty[s]);
         }
@@ -393,31 +376,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     float* stage = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES) + (warp - 2) * C::EPI_STAGE_FLOATS;
     int local = 0;
-    for (int tile = tile_first; tile < tile_last; tile += tile_step, ++local) {
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
       const int b = local & 1, use = local >> 1;
       const int m_tile = tile / num_n, n_tile = tile % num_n;
       const bool ok = mbar_wait(&acc_full[b], use & 1);
       tc_fence_after();
-      if constexpr (SPLIT) {
-        // raw accumulator, chunk-major: [BN/32][128 rows][32]; each lane its row's 128 bytes
-        float* part = g.part + (size_t)blockIdx.x * BM * BN;
-#pragma unroll 1
-        for (int i = 0; i < BN / 64; ++i) {
-          const int c = half * (BN / 2) + 32 * i;
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + b * BN + c, r);
-          tmem_wait_ld();
-          float4* dst = reinterpret_cast<float4*>(part + (size_t)(c / 32) * (BM * 32) + (size_t)(q * 32 + lane) * 32);
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            dst[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
-                                 __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
-        }
-        tc_fence_before();
-        mbar_arrive(&acc_empty[b]);
-        if (!ok) break;
-        continue;
-      }
       const int64_t row0 = (int64_t)m_tile * BM + q * 32;
       // this warp's chunks: columns [half * BN/2, (half + 1) * BN/2) of the tile, 32 at a time;
       // the global inputs of chunk i+1 (residual, bias, gates) are loaded while chunk i is processed
@@ -451,46 +414,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
-}
-
-// The tiles of a split round: adds each tile's K-range parts in split order
-// (the result does not depend on timing) and applies the epilogue of KIND.
-// One CTA per (tile, 64-column slab); warp w takes rows 32 (w % 4) .. +31 and
-// 32-column chunk w / 4 of the slab, the layout of the main kernel's
-// epilogue warps, so the epilogue code is the same.
-template <int BN, int KIND, bool R32>
-__global__ void __launch_bounds__(32 * kEpiWarps) gemm_split_fixup_kernel(GemmDims g, EpiDev e) {
-  extern __shared__ float fixup_stage[];  // kEpiWarps x 32 x 33
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  constexpr int SLABS = BN / 64;
-  const int ti = (int)blockIdx.x / SLABS, slab = (int)blockIdx.x % SLABS;
-  const int tile = g.split_base + ti;
-  const int num_n = (g.N + BN - 1) / BN;
-  const int q = warp & 3, ci = slab * 2 + (warp >> 2);  // 32-column chunk within the tile
-  const int64_t row0 = (int64_t)(tile / num_n) * BM + q * 32;
-  const int col0 = (tile % num_n) * BN + ci * 32;
-  if (row0 >= g.M || col0 >= g.N) return;
-  float acc[32];
-#pragma unroll
-  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
-  for (int sp = 0; sp < g.splits; ++sp) {
-    const float4* src = reinterpret_cast<const float4*>(g.part + (size_t)(ti * g.splits + sp) * BM * BN +
-                                                        (size_t)ci * (BM * 32) + (size_t)(q * 32 + lane) * 32);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float4 v = src[j];
-      acc[4 * j] += v.x;
-      acc[4 * j + 1] += v.y;
-      acc[4 * j + 2] += v.z;
-      acc[4 * j + 3] += v.w;
-    }
-  }
-  uint32_t r[32];
-#pragma unroll
-  for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(acc[j]);
-  ResChunk<R32> rc;
-  load_chunk_inputs<KIND, R32>(g, e, row0, col0 + 4 * (lane & 7), rc);
-  epilogue_chunk<KIND, R32>(g, e, fixup_stage + warp * 32 * 33, row0, col0, r, rc);
 }
 
 // ---------------------------------------------------------------------------
@@ -548,18 +471,9 @@ int num_sms() {
   return n;
 }
 
-// A split round gives each split at least this many 64-wide K blocks
-// (1024 of K).  Measured at 32760 rows: FFN2 (K = 8960, 8 splits) gains,
-// 564 -> 551 us; K = 1536 layers split 3 ways lose (output projection 117 ->
-// 132 us): the extra launches, the pipeline fill of 8 K blocks, the partial
-// stores and the fixup cost more than their short partial round.
-constexpr int kMinSplitKb = 16;
-
-// The persistent launch; with split_grid > 0 (BN = 256 only) also the split
-// round's CTAs and the fixup that adds their parts and applies the epilogue.
 template <int BN, int KIND, bool R32 = false>
 acid_status launch_tc_kind(const CUtensorMap& ta, const CUtensorMap& tb, const GemmDims& g, const Epilogue& epi,
-                           int grid, int split_grid, cudaStream_t s) {
+                           int grid, cudaStream_t s) {
   using C = TcCfg<BN>;
   static bool attr_done = false;
   if (!attr_done) {
@@ -568,22 +482,6 @@ acid_status launch_tc_kind(const CUtensorMap& ta, const CUtensorMap& tb, const G
   }
   gemm_tc_kernel<BN, KIND, R32><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
   ACID_CHECK_LAUNCH();
-  if constexpr (BN == 256) {
-    if (split_grid > 0) {
-      static bool split_attr_done = false;
-      if (!split_attr_done) {
-        ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI_BIAS, false, true>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
-        split_attr_done = true;
-      }
-      gemm_tc_kernel<BN, EPI_BIAS, false, true><<<split_grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, EpiDev{});
-      ACID_CHECK_LAUNCH();
-      const int tiles = split_grid / g.splits;
-      gemm_split_fixup_kernel<BN, KIND, R32>
-          <<<tiles * (BN / 64), 32 * kEpiWarps, kEpiWarps * 32 * 33 * sizeof(float), s>>>(g, to_dev(epi));
-      ACID_CHECK_LAUNCH();
-    }
-  }
   return ACID_OK;
 }
 
@@ -593,38 +491,20 @@ acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* 
   CUtensorMap ta, tb;
   ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
   ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, BN));
+  GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0};
   const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
-  GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0, (int)tiles, 0, 0, nullptr};
-  const int sms = num_sms();
-  const int grid = (int)std::min<int64_t>(tiles, sms);
-  // A partial last round of tiles (tail of them on tail SMs) is split along K
-  // over up to all SMs when scratch is given and each split keeps at least
-  // kMinSplitKb K blocks; the persistent CTAs then take the full rounds only.
-  int split_grid = 0;
-  if constexpr (BN == 256) {
-    const int64_t full = tiles / sms * sms, tail = tiles - full;
-    const int num_kb = (K + BK - 1) / BK;
-    const int splits = tail > 0 ? (int)std::min<int64_t>(sms / tail, num_kb / kMinSplitKb) : 0;
-    if (epi.split_ws != nullptr && full > 0 && tail > 0 && splits >= 2 &&
-        epi.split_ws_bytes >= (size_t)tail * splits * BM * BN * sizeof(float)) {
-      g.tile_end = (int)full;
-      g.split_base = (int)full;
-      g.splits = splits;
-      g.part = epi.split_ws;
-      split_grid = (int)tail * splits;
-    }
-  }
+  const int grid = (int)std::min<int64_t>(tiles, num_sms());
   ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
   switch (epi.kind) {
-    case EPI_GELU: return launch_tc_kind<BN, EPI_GELU>(ta, tb, g, epi, grid, split_grid, s);
-    case EPI_ROPE_QKV: return launch_tc_kind<BN, EPI_ROPE_QKV>(ta, tb, g, epi, grid, split_grid, s);
+    case EPI_GELU: return launch_tc_kind<BN, EPI_GELU>(ta, tb, g, epi, grid, s);
+    case EPI_ROPE_QKV: return launch_tc_kind<BN, EPI_ROPE_QKV>(ta, tb, g, epi, grid, s);
     case EPI_GATED_RES:
-      return epi.res_fp32 ? launch_tc_kind<BN, EPI_GATED_RES, true>(ta, tb, g, epi, grid, split_grid, s)
-                          : launch_tc_kind<BN, EPI_GATED_RES, false>(ta, tb, g, epi, grid, split_grid, s);
+      return epi.res_fp32 ? launch_tc_kind<BN, EPI_GATED_RES, true>(ta, tb, g, epi, grid, s)
+                          : launch_tc_kind<BN, EPI_GATED_RES, false>(ta, tb, g, epi, grid, s);
     case EPI_RES:
-      return epi.res_fp32 ? launch_tc_kind<BN, EPI_RES, true>(ta, tb, g, epi, grid, split_grid, s)
-                          : launch_tc_kind<BN, EPI_RES, false>(ta, tb, g, epi, grid, split_grid, s);
-    default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, g, epi, grid, split_grid, s);
+      return epi.res_fp32 ? launch_tc_kind<BN, EPI_RES, true>(ta, tb, g, epi, grid, s)
+                          : launch_tc_kind<BN, EPI_RES, false>(ta, tb, g, epi, grid, s);
+    default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, g, epi, grid, s);
   }
 }
 

@@ -49,15 +49,7 @@ struct Epilogue {
   int64_t rope_first_video = 0;
   int d = 0, head_dim = 0;
   bool out_fp32 = false;           // output dtype fp32 (else the GEMM dtype)
-  // optional device scratch (kGemmSplitBytes) for splitting the tiles of a
-  // partial last round along K; null runs that round on fewer CTAs
-  float* split_ws = nullptr;
-  size_t split_ws_bytes = 0;
 };
-
-// Scratch that lets a bf16 linear layer split its partial last round of
-// 128 x 256 tiles along K: fp32 partial tiles for up to 160 CTAs.
-constexpr size_t kGemmSplitBytes = (size_t)160 * 128 * 256 * sizeof(float);
 
 // out[M, N] (row stride ldo) = epilogue(A[M, K] (row stride lda) * W[N, K]^T)
 acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int K, const void* W,

@@ -2,7 +2,7 @@
 warm-up), for tuning and for profiler captures of a single launch.
 
     python -m paper_2607_12358_gb300.kernel_bench attention --n 32760 --heads 12 --head-dim 128
-    python -m paper_2607_12358_gb300.kernel_bench linear --m 32760 --k 1536 --n 8960 --epi gelu [--workspace]
+    python -m paper_2607_12358_gb300.kernel_bench linear --m 32760 --k 1536 --n 8960 --epi gelu
     python -m paper_2607_12358_gb300.kernel_bench drift --rows 118800 --cols 3072 [--apply]
     python -m paper_2607_12358_gb300.kernel_bench block --workload wan [--block-type wan]
 
@@ -53,8 +53,6 @@ def main():
     ap.add_argument("--rows", type=int, default=118800)
     ap.add_argument("--cols", type=int, default=3072)
     ap.add_argument("--apply", action="store_true")
-    ap.add_argument("--workspace", action="store_true",
-                    help="linear: pass the split workspace (a partial last round of tiles is split along K)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--iters", type=int, default=5)
     a = ap.parse_args()
@@ -84,11 +82,10 @@ def main():
         gate = torch.randn(a.n, device=dev, generator=gen)
         y = torch.randn(a.m, a.n, device=dev, generator=gen).to(torch.bfloat16)
         res = y if a.epi in ("gated_res", "res") else None
-        ws = torch.empty(acid.linear_workspace_size(), dtype=torch.uint8, device=dev) if a.workspace else None
-        ms = _time(lambda: acid.acid_linear_forward(x, wt, b, epilogue=a.epi, gate=gate, residual=res, out=y,
-                                                    workspace=ws), a.warmup, a.iters)
+        ms = _time(lambda: acid.acid_linear_forward(x, wt, b, epilogue=a.epi, gate=gate, residual=res, out=y),
+                   a.warmup, a.iters)
         flop = 2.0 * a.m * a.n * a.k
-        out.update(shape=[a.m, a.k, a.n], epi=a.epi, workspace=a.workspace, ms=ms, tflops=flop / ms / 1e9)
+        out.update(shape=[a.m, a.k, a.n], epi=a.epi, ms=ms, tflops=flop / ms / 1e9)
     elif a.kernel == "block":
         import acid_synth as S
 

@@ -112,7 +112,7 @@ def test_host_validation_without_gpu(lib):
     # the failure-path diagnostic validates its budget before launching anything
     assert lib.acid_selftest_wait_timeout(10, None) == A.ACID_ERR_INVALID_ARG
     assert lib.acid_linear_forward(A.ACID_BF16, None, 64, 10, 64, None, None, 64, None, 64, 9, None, None, 0, 0,
-                                   None, 0, None) == A.ACID_ERR_INVALID_ARG
+                                   None) == A.ACID_ERR_INVALID_ARG
     # zero rows are a valid empty call (no launch, null pointers allowed);
     # negative rows or an empty key set are not
     for nq, nk, want in ((0, 4, A.ACID_OK), (-1, 4, A.ACID_ERR_INVALID_ARG), (0, 0, A.ACID_ERR_INVALID_ARG)):
@@ -120,7 +120,7 @@ def test_host_validation_without_gpu(lib):
                                           None, 0, None) == want
     for M, want in ((0, A.ACID_OK), (-1, A.ACID_ERR_INVALID_ARG), (4, A.ACID_ERR_INVALID_ARG)):
         assert lib.acid_linear_forward(A.ACID_BF16, None, 64, M, 64, None, None, 64, None, 64, A.ACID_EPI_BIAS,
-                                       None, None, 0, 0, None, 0, None) == want
+                                       None, None, 0, 0, None) == want
     n = ctypes.c_size_t()
     assert lib.acid_attention_workspace_size(128, ctypes.byref(n)) == A.ACID_OK and n.value > 0
 

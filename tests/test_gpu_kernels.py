@@ -126,66 +126,6 @@ def test_linear_bf16_partial_last_column_tile(acid, M, K, N, epi):
     assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
 
 
-def _split_round(M, N, sms):
-    """Element mask and rows of the tiles of the partial last round (128 x 256
-    tiles numbered with N fastest, sms persistent CTAs)."""
-    num_n = -(-N // 256)
-    tiles = -(-M // 128) * num_n
-    full = tiles // sms * sms
-    mask = np.zeros((M, N), dtype=bool)
-    for t in range(full, tiles):
-        mt, nt = divmod(t, num_n)
-        mask[mt * 128:(mt + 1) * 128, nt * 256:(nt + 1) * 256] = True
-    return mask, np.flatnonzero(mask.any(axis=1)), tiles - full
-
-
-@pytest.mark.parametrize("M,K,N", [(20000, 4096, 256), (19500, 3072, 1536), (3584, 8960, 1536)])
-@pytest.mark.parametrize("epi,fp32", [("bias", False), ("gelu", False), ("gated_res", True), ("gated_res", False),
-                                      ("res", True)])
-def test_linear_split_last_round(acid, M, K, N, epi, fp32):
-    """With a workspace, the tiles of a partial last round run split along K
-    over all SMs, and a fixup adds the parts in a fixed order before the
-    epilogue.  Cases: 5 tail tiles over 4 splits; a ragged 44-row last row
-    block over 3 splits; 16 tail tiles over 8 splits (the FFN2 pattern at
-    K = 8960).  Every row that touches a split tile and a sample of the
-    others match the oracle; two runs are bit-identical; tiles outside the
-    split round equal the unsplit launch bit for bit, and the split tiles
-    equal it up to summation order."""
-    sms = torch.cuda.get_device_properties(0).multi_processor_count
-    mask, rows_tail, tail = _split_round(M, N, sms)
-    assert tail > 0
-    rng = np.random.default_rng(M + K + N)
-    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
-    w = S.round_to_bf16((0.05 * rng.normal(size=(N, K))).astype(np.float32))
-    b = rng.normal(size=N).astype(np.float32)
-    g = rng.normal(size=N).astype(np.float32)
-    r = rng.normal(size=(M, N)).astype(np.float32)
-    if not fp32:
-        r = S.round_to_bf16(r)
-    has_res = epi in ("gated_res", "res")
-    ws = torch.empty(acid.linear_workspace_size(), dtype=torch.uint8, device=DEV)
-    ta, tw, tb, tg = _bf(a), _bf(w), _f32(b), _f32(g)
-
-    def run(workspace):
-        res = (_f32(r) if fp32 else _bf(r)) if has_res else None
-        out = acid.acid_linear_forward(ta, tw, tb, epilogue=epi, gate=tg, residual=res, out=res, out_fp32=fp32,
-                                       workspace=workspace)
-        torch.cuda.synchronize()
-        return out.float().cpu().numpy()
-
-    split1, split2, plain = run(ws), run(ws), run(None)
-    acid.check_device_error()
-    np.testing.assert_array_equal(split1, split2)
-    np.testing.assert_array_equal(split1[~mask], plain[~mask])
-    rows = np.unique(np.concatenate([rows_tail, np.arange(0, M, max(1, M // 100))]))
-    acc = O.linear(a[rows], w, b)
-    rr = r[rows]
-    ref = {"bias": acc, "gelu": O.gelu_tanh(acc), "gated_res": rr + g * acc, "res": rr + acc}[epi]
-    tol = 1e-4 if (fp32 and epi != "gelu") else 2 ** -8
-    assert np.abs(split1[rows] - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(split1[rows] - ref).max()
-    assert np.abs(split1[mask] - plain[mask]).max() <= tol * (np.abs(plain).max() + 1)
-
-
 @pytest.mark.parametrize("M,K,N", [(1, 64, 64), (7, 8, 32), (127, 72, 96), (129, 200, 256), (3, 4104, 128)])
 def test_linear_bf16_edge_shapes(acid, M, K, N):
     """Single rows, K below / not a multiple of the 64-wide k-block (zero-filled
