@@ -106,3 +106,24 @@ def test_bf16_graph_equals_host_loop(acid, kind):
     host, graph, la, lb = _both(acid, cfg, w, S.latent(cfg, 7), S.text(cfg, 7), **kw)
     _same_logs(la, lb)
     np.testing.assert_array_equal(graph, host)
+
+
+def test_graph_at_its_step_limit(acid):
+    """The graph keeps its per-step tables (noise levels, forced decisions,
+    thresholds, logs) for at most 1024 steps: a 1024-step generation runs as
+    one graph and equals the host-driven loop bit for bit, decisions
+    included; 1025 steps are refused before anything is launched."""
+    from paper_2607_12358_gb300._capi import AcidError
+
+    cfg = S.get_config("toy", steps=1024)
+    w = S.model_weights(cfg, 60)
+    a, b, la, lb = _both(acid, cfg, w, S.latent(cfg, 60))
+    _same_logs(la, lb)
+    np.testing.assert_array_equal(a, b)
+    assert len(lb) == 1024 and 0 < sum(l["computed"] for l in lb) < 1024
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg, n_steps=1025)
+    n0 = acid.launch_count()
+    with pytest.raises(AcidError, match="at most 1024 steps"):
+        acid.acid_denoise_loop(model, c, torch.from_numpy(S.latent(cfg, 60)).to(DEV), None, graph=True)
+    assert acid.launch_count() == n0
