@@ -223,6 +223,25 @@ def test_attention_persistent_items(acid, nq, nk, H, D):
         assert np.abs(got - ref).max() <= 5e-2, (w is None, np.abs(got - ref).max())
 
 
+@pytest.mark.parametrize("nq,nk,H,D", [(131072, 512, 12, 128), (65536, 500, 24, 64)])
+def test_attention_persistent_many_items(acid, nq, nk, H, D):
+    """Long runs of items per persistent CTA: 6144 items over 152 CTAs (about
+    40 each, 160 key-tile steps whose barrier phases and ring slots carry
+    across items) at head dim 128, and over 304 CTAs (about 20 each, masked
+    last tile) at head dim 64.  Sampled rows, the first and last items among
+    them, against the oracle."""
+    rng = np.random.default_rng(nq + nk)
+    q = S.round_to_bf16((2.0 * rng.standard_normal(size=(nq, H * D), dtype=np.float32)))
+    k = S.round_to_bf16(rng.standard_normal(size=(nk, H * D), dtype=np.float32))
+    v = S.round_to_bf16(rng.standard_normal(size=(nk, H * D), dtype=np.float32))
+    got = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), H).float().cpu().numpy()
+    acid.check_device_error()
+    rows = np.unique(np.concatenate([np.arange(0, 300), np.arange(0, nq, nq // 97), np.arange(nq - 300, nq)]))
+    ref = O.attention(q[rows].reshape(-1, H, D), k.reshape(nk, H, D), v.reshape(nk, H, D)).reshape(len(rows), H * D)
+    assert _rel_l2(got[rows], ref) <= 1e-2, _rel_l2(got[rows], ref)
+    assert np.abs(got[rows] - ref).max() <= 5e-2
+
+
 def test_attention_one_key_returns_value(acid):
     q, k, v, ref = _attn_case(200, 1, 2, 128, 3)
     got = acid.acid_attention_forward(_bf(q), _bf(k), _bf(v), 2).float().cpu().numpy()
