@@ -247,12 +247,6 @@ def model_weights(cfg: DiTConfig, seed: int = 0, blocks: bool = True) -> dict:
     return m
 
 
-def block_types(cfg: DiTConfig) -> list[str]:
-    if cfg.kind == "hv":
-        return ["hv_dual"] * cfg.n_blocks + ["hv_single"] * cfg.n_single
-    return [cfg.kind] * cfg.n_blocks
-
-
 # ----------------------------------------------------------------------------
 # Activations and inputs.
 # ----------------------------------------------------------------------------
