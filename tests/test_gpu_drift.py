@@ -133,3 +133,49 @@ def test_drift_rejects_small_workspace(acid):
     a = torch.zeros(64, device=DEV, dtype=torch.bfloat16)
     with pytest.raises(AcidError):
         acid.acid_drift_signal(a, a, workspace=torch.empty(16, dtype=torch.uint8, device=DEV))
+
+
+def test_drift_and_apply_past_32_bit_offsets(acid):
+    """2^31 + 13 bf16 elements (4.3 GB per tensor): element offsets past 2^31,
+    byte offsets past 4 GiB and a ragged tail of 5 after the last 8-wide vector.
+
+    prev_i = 1 + (i mod 7), cur = 1.25 prev and residual_i = (i mod 5)/2 - 1.
+    Every value, difference and per-thread fp32 partial sum is a multiple of
+    1/4 far below 2^22, so all of them are exact in bf16 and fp32.
+    Hence rel_l1 = 1/4 exactly, Σ|prev| = 28 q + r(r+1)/2 with n = 7q + r,
+    and out = cur + residual holds element for element, by the plain cache
+    apply and by the fused drift + apply alike."""
+    n = 2 ** 31 + 13
+    chunk = 2 ** 28
+    prev = torch.empty(n, dtype=torch.bfloat16, device=DEV)
+    cur = torch.empty_like(prev)
+    res = torch.empty_like(prev)
+    for s in range(0, n, chunk):
+        i = torch.arange(s, min(n, s + chunk), device=DEV, dtype=torch.int64)
+        p = (1 + i % 7).to(torch.float32)
+        prev[s:s + i.numel()] = p.to(torch.bfloat16)
+        cur[s:s + i.numel()] = (1.25 * p).to(torch.bfloat16)
+        res[s:s + i.numel()] = ((i % 5).to(torch.float32) * 0.5 - 1.0).to(torch.bfloat16)
+        del i, p
+    q, r = divmod(n, 7)
+    den = 28 * q + r * (r + 1) // 2
+
+    rel, sums = acid.acid_drift_signal(prev, cur)
+    assert rel.item() == 0.25
+    assert sums.cpu().tolist() == [den / 4, float(den)]
+
+    def check_out(out):
+        for s in range(0, n, chunk):
+            i = torch.arange(s, min(n, s + chunk), device=DEV, dtype=torch.int64)
+            want = (1.25 * (1 + i % 7).to(torch.float32) + (i % 5).to(torch.float32) * 0.5 - 1.0).to(torch.bfloat16)
+            assert torch.equal(out[s:s + i.numel()], want), f"chunk at {s}"
+            del i, want
+
+    out = acid.acid_cache_apply(cur, res)
+    check_out(out)
+    out.zero_()
+    out, rel2, sums2 = acid.acid_drift_apply(prev, cur, res, out=out)
+    assert rel2.item() == 0.25 and sums2.cpu().tolist() == [den / 4, float(den)]
+    check_out(out)
+    del prev, cur, res, out
+    torch.cuda.empty_cache()

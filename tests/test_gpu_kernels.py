@@ -126,6 +126,38 @@ def test_linear_bf16_partial_last_column_tile(acid, M, K, N, epi):
     assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
 
 
+def test_linear_bf16_offsets_past_32_bits(acid):
+    """An output of 262181 x 8960 fp32 values (2.35e9 elements, 9.4 GB),
+    updated in place by the gated-residual epilogue.  Rows from 239675 on
+    start past element 2^31, so the residual reads and the stores there need
+    64-bit offsets; the last row tile holds 37 rows.  Sampled rows, at both
+    ends and around the 2^31 boundary, are compared with the oracle."""
+    M, K, N = 262144 + 37, 64, 8960
+    rng = np.random.default_rng(31)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.1 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    g = rng.normal(size=N).astype(np.float32)
+
+    def resid(rows):  # a closed-form residual, cheap to build on the device and on the host
+        return ((rows[:, None] * 7 + np.arange(N)[None, :]) % 13).astype(np.float32) / 4 - 1.5
+
+    res = torch.empty((M, N), dtype=torch.float32, device=DEV)
+    cols = torch.arange(N, device=DEV, dtype=torch.int64)
+    for r0 in range(0, M, 16384):
+        rows = torch.arange(r0, min(M, r0 + 16384), device=DEV, dtype=torch.int64)
+        res[r0:r0 + rows.numel()] = ((rows[:, None] * 7 + cols[None, :]) % 13).float() / 4 - 1.5
+        del rows
+    out = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), epilogue="gated_res", gate=_f32(g), residual=res,
+                                   out=res, out_fp32=True)
+    rows = np.array([0, 1, 127, 128, 239674, 239675, 239676, 262015, 262143, 262144, 262180])
+    got = out[torch.from_numpy(rows).to(DEV)].cpu().numpy()
+    ref = resid(rows) + g * O.linear(a[rows], w, b)
+    assert np.abs(got - ref).max() <= 1e-4 * (np.abs(ref).max() + 1), np.abs(got - ref).max()
+    del res, out
+    torch.cuda.empty_cache()
+
+
 @pytest.mark.parametrize("M,K,N", [(1, 64, 64), (7, 8, 32), (127, 72, 96), (129, 200, 256), (3, 4104, 128)])
 def test_linear_bf16_edge_shapes(acid, M, K, N):
     """Single rows, K below / not a multiple of the 64-wide k-block (zero-filled
