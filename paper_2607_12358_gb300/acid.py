@@ -179,10 +179,13 @@ def acid_attention_forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, he
 
 
 def acid_layernorm_mod(x: torch.Tensor, shift: torch.Tensor | None = None, scale: torch.Tensor | None = None,
-                       eps: float = 1e-6, out_dtype=None, stream=None) -> torch.Tensor:
-    """y = LN(x) * (1 + scale) + shift over the last axis of x [rows, d]."""
-    _need_cuda(x, shift, scale)
-    y = torch.empty(x.shape, dtype=out_dtype or x.dtype, device=x.device)
+                       eps: float = 1e-6, out_dtype=None, stream=None, out: torch.Tensor | None = None) -> torch.Tensor:
+    """y = LN(x) * (1 + scale) + shift over the last axis of x [rows, d]
+    (written into `out` when given: same shape, dtype out_dtype or x's)."""
+    _need_cuda(x, shift, scale, out)
+    y = torch.empty(x.shape, dtype=out_dtype or x.dtype, device=x.device) if out is None else out
+    if y.shape != x.shape or not y.is_contiguous():
+        raise ValueError("out must be contiguous with the shape of x")
     check(load().acid_layernorm_mod(_dtype(x), x.data_ptr(), _dtype(y), y.data_ptr(), x.shape[0], x.shape[1],
                                     _ptr(shift), _ptr(scale), eps, _stream(stream)))
     return y

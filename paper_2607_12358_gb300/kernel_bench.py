@@ -4,6 +4,7 @@ warm-up), for tuning and for profiler captures of a single launch.
     python -m paper_2607_12358_gb300.kernel_bench attention --n 32760 --heads 12 --head-dim 128
     python -m paper_2607_12358_gb300.kernel_bench linear --m 32760 --k 1536 --n 8960 --epi gelu
     python -m paper_2607_12358_gb300.kernel_bench drift --rows 118800 --cols 3072 [--apply]
+    python -m paper_2607_12358_gb300.kernel_bench layernorm --rows 32760 --cols 1536 --in-dtype fp32
     python -m paper_2607_12358_gb300.kernel_bench block --workload wan [--block-type wan]
 
 Inputs are random bf16 tensors created on the device (block: the synthetic
@@ -40,7 +41,7 @@ def _time(fn, warmup, iters):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attention", "linear", "drift", "block"])
+    ap.add_argument("kernel", choices=["attention", "linear", "drift", "layernorm", "block"])
     ap.add_argument("--workload", default="wan", help="block: wan | cog | hv")
     ap.add_argument("--block-type", default=None, help="block: wan | cog | hv_dual | hv_single")
     ap.add_argument("--n", type=int, default=32760)
@@ -53,6 +54,7 @@ def main():
     ap.add_argument("--rows", type=int, default=118800)
     ap.add_argument("--cols", type=int, default=3072)
     ap.add_argument("--apply", action="store_true")
+    ap.add_argument("--in-dtype", default="bf16", choices=["bf16", "fp32"], help="layernorm: input dtype")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--iters", type=int, default=5)
     a = ap.parse_args()
@@ -86,6 +88,18 @@ def main():
                    a.warmup, a.iters)
         flop = 2.0 * a.m * a.n * a.k
         out.update(shape=[a.m, a.k, a.n], epi=a.epi, ms=ms, tflops=flop / ms / 1e9)
+    elif a.kernel == "layernorm":
+        # adaLN LayerNorm of the residual stream into the bf16 GEMM operand:
+        # reads x once, writes y once (the shift / scale vectors stay in L2)
+        dt = torch.float32 if a.in_dtype == "fp32" else torch.bfloat16
+        x = torch.randn(a.rows, a.cols, device=dev, generator=gen).to(dt)
+        shift = torch.randn(a.cols, device=dev, generator=gen)
+        scale = torch.randn(a.cols, device=dev, generator=gen)
+        y = torch.empty(a.rows, a.cols, device=dev, dtype=torch.bfloat16)
+        ms = _time(lambda: acid.acid_layernorm_mod(x, shift, scale, out_dtype=torch.bfloat16, out=y),
+                   a.warmup, a.iters)
+        nbytes = float(a.rows) * a.cols * (x.element_size() + 2)
+        out.update(shape=[a.rows, a.cols], in_dtype=a.in_dtype, ms=ms, gbs=nbytes / ms / 1e6)
     elif a.kernel == "block":
         import acid_synth as S
 

@@ -336,6 +336,22 @@ def test_layernorm_mod(acid, d):
     assert np.abs(got16 - ref).max() <= 2 ** -8 * (1 + np.abs(ref).max())
 
 
+@pytest.mark.parametrize("d", [1536, 3072])
+def test_layernorm_mod_fp32_input_into_bf16_buffer(acid, d):
+    """The block's case: the fp32 residual stream normalised into a bf16 GEMM
+    operand, written into a caller-given buffer (one bf16 rounding of the
+    fp64 reference)."""
+    rng = np.random.default_rng(d + 1)
+    x = (0.5 + 4.0 * rng.normal(size=(1001, d))).astype(np.float32)
+    sh, sc = rng.normal(size=d).astype(np.float32), rng.normal(size=d).astype(np.float32)
+    ref = O.modulate(O.layer_norm(x), sh, sc)
+    y = torch.full((1001, d), float("nan"), dtype=torch.bfloat16, device=DEV)
+    got = acid.acid_layernorm_mod(_f32(x), _f32(sh), _f32(sc), out_dtype=torch.bfloat16, out=y)
+    assert got.data_ptr() == y.data_ptr()
+    got = got.float().cpu().numpy()
+    assert np.abs(got - ref).max() <= 2 ** -8 * (1 + np.abs(ref).max())
+
+
 def test_empty_inputs_return_without_launching(acid):
     """Zero rows: the linear layer, attention, LayerNorm-mod and cache apply
     return OK and launch nothing."""
