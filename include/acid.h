@@ -23,6 +23,12 @@
  *    acid_last_error() gives a message (thread-local).
  *  - Device-side waits are bounded.  A wait that runs out sets a device flag
  *    that acid_check_device_error() reports as ACID_ERR_TIMEOUT.
+ *  - One CUDA device per process.  The kernels' shared-memory attributes and
+ *    the SM count used to size persistent grids are set up at the first call,
+ *    for the device current then.  Several GPUs are served by one process
+ *    each; a call on another device of the same process may fail with
+ *    ACID_ERR_CUDA.  Calls that share a workspace must be ordered by their
+ *    streams.
  */
 #ifndef ACID_H_
 #define ACID_H_
