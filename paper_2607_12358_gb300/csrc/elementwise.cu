@@ -285,11 +285,18 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
 // step_dev is given (graph-launched loops), else step_host is used.  At step
 // 0 there is no previous TEMNI and the sums are zero.  One warp per row
 // (grid-strided), fp64 CTA partials reduced by drift_final_kernel.
-__global__ void __launch_bounds__(kThreads) ln_mod_drift_kernel(const float* __restrict__ x, float* tem0, float* tem1,
-                                                                const int* step_dev, int step_host, int64_t rows, int d,
-                                                                const float* __restrict__ shift,
-                                                                const float* __restrict__ scale, float eps,
-                                                                double2* __restrict__ partials) {
+// NV: 8-element vectors per lane (d <= 256 * NV), so that the row held in
+// registers is sized to d.  For rows up to 1536 wide the previous TEMNI row
+// is loaded together with x: a row then costs one DRAM round trip, not two.
+// The arithmetic and its order do not depend on NV.
+template <int NV>
+__global__ void __launch_bounds__(kThreads, 2) ln_mod_drift_kernel(const float* __restrict__ x, float* tem0,
+                                                                   float* tem1, const int* step_dev, int step_host,
+                                                                   int64_t rows, int d,
+                                                                   const float* __restrict__ shift,
+                                                                   const float* __restrict__ scale, float eps,
+                                                                   double2* __restrict__ partials) {
+  constexpr bool kPrevEarly = NV <= 6;
   const int step = step_dev ? *step_dev : step_host;
   float* cur = (step & 1) ? tem1 : tem0;
   const float* prev = (step & 1) ? tem0 : tem1;
@@ -300,13 +307,24 @@ __global__ void __launch_bounds__(kThreads) ln_mod_drift_kernel(const float* __r
   float num = 0.f, den = 0.f;
   for (int64_t row = gw; row < rows; row += nw) {
     const float* xr = x + row * d;
-    float v[kLnMaxV][8];
-    float s = 0.f;
+    const float* pr = prev + row * d;
+    float v[NV][8];
+    float pe[kPrevEarly ? NV : 1][8];
 #pragma unroll
-    for (int i = 0; i < kLnMaxV; ++i) {
+    for (int i = 0; i < NV; ++i) {
       const int c = (i * 32 + lane) * 8;
       if (c < d) {
         load8(xr + c, v[i]);
+        if constexpr (kPrevEarly) {
+          if (has_prev) load8(pr + c, pe[i]);
+        }
+      }
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      const int c = (i * 32 + lane) * 8;
+      if (c < d) {
 #pragma unroll
         for (int j = 0; j < 8; ++j) s += v[i][j];
       }
@@ -314,7 +332,7 @@ __global__ void __launch_bounds__(kThreads) ln_mod_drift_kernel(const float* __r
     const float mean = warp_sum_f(s) / d;
     float q = 0.f;
 #pragma unroll
-    for (int i = 0; i < kLnMaxV; ++i) {
+    for (int i = 0; i < NV; ++i) {
       const int c = (i * 32 + lane) * 8;
       if (c < d) {
 #pragma unroll
@@ -326,18 +344,24 @@ __global__ void __launch_bounds__(kThreads) ln_mod_drift_kernel(const float* __r
     }
     const float rstd = rsqrtf(warp_sum_f(q) / d + eps);
 #pragma unroll
-    for (int i = 0; i < kLnMaxV; ++i) {
+    for (int i = 0; i < NV; ++i) {
       const int c = (i * 32 + lane) * 8;
       if (c < d) {
-        float a[8], b[8], o[8];
+        float a[8], b[8];
         load8(scale + c, a);
         load8(shift + c, b);
+        float* o = v[i];  // the output replaces the input in place
 #pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = fmaf((v[i][j] - mean) * rstd, 1.0f + a[j], b[j]);
+        for (int j = 0; j < 8; ++j) o[j] = fmaf((o[j] - mean) * rstd, 1.0f + a[j], b[j]);
         store8(cur + row * d + c, o);
         if (has_prev) {
-          float p[8];
-          load8(prev + row * d + c, p);
+          float pl[kPrevEarly ? 1 : 8];
+          const float* p = pl;
+          if constexpr (kPrevEarly) {
+            p = pe[i];
+          } else {
+            load8(pr + c, pl);
+          }
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             num += fabsf(o[j] - p[j]);
@@ -617,7 +641,15 @@ acid_status ln_mod_drift(const float* x, float* tem0, float* tem1, const int* st
   const int64_t want = (rows * 32 + kThreads - 1) / kThreads;
   const int grid = (int)std::min<int64_t>(kDriftMaxBlocks, std::max<int64_t>(1, want));
   ProfScope prof(PROF_DRIFT, (double)rows * d * 12.0, s);  // read x and prev, write cur (fp32)
-  ln_mod_drift_kernel<<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
+  if (d <= 256 * 4)
+    ln_mod_drift_kernel<4><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
+  else if (d <= 256 * 6)
+    ln_mod_drift_kernel<6><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
+  else if (d <= 256 * 8)
+    ln_mod_drift_kernel<8><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
+  else
+    ln_mod_drift_kernel<kLnMaxV><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale,
+                                                           eps, parts);
   ACID_CHECK_LAUNCH();
   drift_final_kernel<<<1, kThreads, 0, s>>>(parts, grid, d_result);
   ACID_CHECK_LAUNCH();
