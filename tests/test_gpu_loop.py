@@ -217,3 +217,34 @@ def test_bf16_loop_teacher_forced_signal_and_replay(acid, kind):
     assert dec == [bool(l["computed"]) for l in logs]
     assert all(math.isfinite(l["signal"]) for l in logs[W:])
     assert np.isfinite(tl.cpu().numpy()).all()
+
+
+@pytest.mark.parametrize("d", [1024, 1152, 1920, 2048, 2560])
+def test_teacache_signal_across_row_widths(acid, d):
+    """The fused TEMNI + drift kernel keeps the row in registers sized to the
+    width (up to 1024, 1536, 2048 or 3072 columns; up to 1536 it also loads
+    the previous TEMNI row with the input).  The toy, Wan and HunyuanVideo
+    loops cover widths 256, 1536 and 3072.  Here the edges of the ranges and
+    the CogVideoX width 1920 (its last vector half filled) run TeaCache, and
+    the loop's signal matches the oracle's relative L1 of consecutive TEMNIs,
+    teacher-forced on the GPU's own step inputs."""
+    cfg = S.get_config("wan", d=d, heads=d // 128, ffn=512, n_blocks=1, n_text=40, d_text=256, latent_f=3,
+                       latent_h=16, latent_w=22, steps=4)
+    w = S.model_weights(cfg, 6)
+    lat = S.latent(cfg, 6)
+    text = S.text(cfg, 6)
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg)
+    loop = acid.Loop(model, c, torch.from_numpy(text).to(DEV, torch.bfloat16), DEV)
+    tl = torch.from_numpy(lat).to(DEV)
+    xs, logs = [], []
+    for i in range(cfg.steps):
+        xs.append(tl.cpu().numpy().astype(np.float64))
+        logs.append(acid.log_to_dict(loop.step(tl)))
+    acid.check_device_error()
+    sig = O.sigmas(cfg.steps)
+    temni = [O.block0_temni(cfg, w, O.step_inputs(cfg, w, x, 1000 * sig[i], with_blocks=False).h_in,
+                            O.time_embedding(1000 * sig[i], w, cfg.time_freq_dim)) for i, x in enumerate(xs)]
+    for i in range(cfg.warmup, cfg.steps):
+        ref = O.rel_l1(temni[i - 1], temni[i])
+        assert abs(logs[i]["signal"] - ref) <= 1e-3 * ref, (d, i, logs[i]["signal"], ref)
