@@ -336,6 +336,7 @@ def run_ours(args) -> None:
     peak = peaks["bf16_tflops_sustained"]
     att_tflops = a_flop / (a_ms / 1000.0) / 1e12 if a_ms > 0 else 0.0
     lin_tflops = l_flop / (l_ms / 1000.0) / 1e12 if l_ms > 0 else 0.0
+    d_gbs = d_bytes / (d_ms / 1000.0) / 1e9 if d_ms > 0 else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -351,7 +352,9 @@ def run_ours(args) -> None:
         "attention_tflops": att_tflops,
         "attention_pct_bf16_peak": 100.0 * att_tflops / peaks["bf16_tflops"],
         "linear": {"tflops": lin_tflops, "launches": l_n, "ms": l_ms},
-        "drift": {"gbs": d_bytes / (d_ms / 1000.0) / 1e9 if d_ms > 0 else None, "launches": d_n, "ms": d_ms},
+        "drift": {"kernel": "ln_mod_drift_kernel (TEMNI and its drift in one pass) + drift_final_kernel",
+                  "gbs": d_gbs, "frac_of_hbm": d_gbs / peaks["hbm_gbs"] if d_gbs else None,
+                  "hbm_peak_source": f"hbm_gbs, {src}", "launches": d_n, "ms": d_ms},
         "block_ms": t_max / K / cfg.n_blocks,
         "acid_mode": {"steps_per_s": K / (acid_ms / 1000.0), "computed_steps": computed, "of": K,
                       "tau_low": cfg.tau_low, "tau_high": cfg.tau_high, "delta": cfg.delta,
