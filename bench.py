@@ -343,7 +343,7 @@ def run_ours(args) -> None:
         "dtype": "bf16", "data": "synthetic (random N(0,0.02) weights, N(0,1) latent and text)",
         "config": {"workload": WORKLOAD, "global_batch": 1, "seq_len": cfg.n_video, "parallelism": "replicas",
                    "schedule": "every step computed (tau_low = tau_high = -1); drift and decision still run",
-                   "l2": "no flush: per-step working set (2.8 GB weights, >0.5 GB activations) exceeds the 129 MB L2"},
+                   "l2": "no flush: per-step working set (3.4 GB of bf16 weights read once per step, >0.5 GB activations) exceeds the 129 MB L2"},
         "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel<128> (self) + attn_persist_kernel<128> (cross attention)",
                      "achieved": att_tflops, "peak": peak, "unit": "TFLOP/s", "frac": att_tflops / peak,
                      "peak_source": f"bf16_tflops_sustained, {src}", "traffic": _attn_traffic(),
