@@ -135,6 +135,25 @@ MUTANTS = [
        "        si = step_inputs(cfg, w, x, sig[i])\n        f = _step_override(forced, i)")], [C], "loop"),
     ("force_last ignored",
      [("if force_last and i == n_steps - 1 and f is None:", "if False:")], [C], "force_last"),
+    ("time MLP without its SiLU",
+     [('    return linear(silu(h), *w["time2"])', '    return linear(h, *w["time2"])')], [P], "silu_closed"),
+    ("block modulation without its SiLU",
+     [("    return linear(silu(temb), *wb)", "    return linear(temb, *wb)")], [P], "silu_closed"),
+    ("final layer with shift and scale swapped",
+     [("final_mod[:d], final_mod[d:])", "final_mod[d:], final_mod[:d])")], [P], "final_layer_on_constant"),
+    ("patch embedding without its bias",
+     [('cfg.pw), *w["patch"])', 'cfg.pw), w["patch"][0])')], [P], "patch_embedding_bias"),
+    ("noise-level shift inverted",
+     [("        s = shift * s / (1.0 + (shift - 1.0) * s)", "        s = s / (shift - (shift - 1.0) * s)")],
+     [P], "sigma_shift"),
+    ("dual-stream text QKV from the video weights",
+     [('    qkv_t = linear(ut, *w["txt.qkv"])', '    qkv_t = linear(ut, *w["vid.qkv"])')], [P], "interchangeable"),
+    ("dual-stream text residual gated by the video gate",
+     [('    yt = xt[rt] + mt[2] * linear(at, *w["txt.o"])', '    yt = xt[rt] + mv[2] * linear(at, *w["txt.o"])')],
+     [P], "interchangeable"),
+    ("dual-stream video FFN input on the text modulation",
+     [("    hv = modulate(layer_norm(yv, eps), mv[3], mv[4])", "    hv = modulate(layer_norm(yv, eps), mt[3], mt[4])")],
+     [P], "interchangeable"),
     ("guidance extrapolates from the conditional branch",
      [("return v_uncond + scale * (v_cond - v_uncond)", "return v_cond + scale * (v_uncond - v_cond)")],
      [G], "guidance or unit_and_zero"),

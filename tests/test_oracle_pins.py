@@ -224,6 +224,61 @@ def test_patchify_matches_conv3d_flatten():
     np.testing.assert_allclose(out, ref, atol=1e-12)
 
 
+def test_time_mlp_and_modulation_silu_closed_forms():
+    """SiLU(ln 3) = ln 3 / (1 + 1/3) = 0.75 ln 3.  A time MLP whose first layer
+    has zero weights and bias ln 3, followed by an identity layer, returns
+    0.75 ln 3 in every unit at any t; the block modulation W SiLU(temb) + b
+    with W = I, b = 0 at temb = ln 3 returns the same."""
+    d, l3 = 6, math.log(3.0)
+    w = {"time1": (np.zeros((d, 256)), np.full(d, l3)), "time2": (np.eye(d), np.zeros(d))}
+    for t in (0.0, 417.0, 1000.0):
+        np.testing.assert_allclose(O.time_embedding(t, w, 256), 0.75 * l3, rtol=1e-15)
+    np.testing.assert_allclose(O.block_modulation(np.full(d, l3), (np.eye(d), np.zeros(d))), 0.75 * l3,
+                               rtol=1e-15)
+
+
+def test_patch_embedding_bias_and_feature_selection():
+    """A zero patch weight leaves its bias on every token; a weight that picks
+    patch feature j reproduces column j of the patchified latent."""
+    cfg = S.get_config("toy")
+    w = S.model_weights(cfg, 0, blocks=False)
+    lat = S.latent(cfg, 0)
+    b = 0.01 * np.arange(cfg.d, dtype=float)
+    h = O.step_inputs(cfg, dict(w, patch=(np.zeros((cfg.d, cfg.patch_dim)), b)), lat, 500.0, with_blocks=False).h_in
+    assert h.shape == (cfg.n_video, cfg.d)
+    np.testing.assert_array_equal(h, np.broadcast_to(b, h.shape))
+    sel = np.zeros((cfg.d, cfg.patch_dim))
+    sel[:, 5] = 1.0
+    h = O.step_inputs(cfg, dict(w, patch=(sel, None)), lat, 500.0, with_blocks=False).h_in
+    np.testing.assert_array_equal(h, np.repeat(O.patchify(lat, 1, 2, 2)[:, 5:6], cfg.d, axis=1))
+
+
+def test_final_layer_on_constant_rows():
+    """A constant row normalises to zero, so the final adaLN leaves only the
+    shift: with every output unit averaging its input, every latent value is
+    mean(shift_f) + bias whatever scale_f is (shift 2, scale 5, bias 0.25
+    give 2.25)."""
+    cfg = S.get_config("toy")
+    d = cfg.d
+    w = {"final": (np.full((cfg.patch_dim, d), 1.0 / d), np.full(cfg.patch_dim, 0.25))}
+    h = np.repeat(np.arange(cfg.n_video, dtype=float)[:, None] - 7.0, d, axis=1)
+    v = O.final_layer(cfg, w, h, np.concatenate([np.full(d, 2.0), np.full(d, 5.0)]))
+    assert v.shape == cfg.latent_shape
+    np.testing.assert_allclose(v, 2.25, rtol=1e-14)
+
+
+def test_sigma_shift_closed_form_and_direction():
+    """sigma' = s sigma / (1 + (s - 1) sigma) keeps 0 and 1, raises every
+    interior level for s > 1 (more of the schedule at high noise) and lowers
+    it for s < 1.  s = 3 on a 4-step grid gives 1, 0.9, 0.75, 0.5, 0."""
+    np.testing.assert_allclose(O.sigmas(4, 3.0), [1.0, 0.9, 0.75, 0.5, 0.0], rtol=1e-15)
+    base = O.sigmas(10)
+    for shift in (1.5, 3.0, 7.0):
+        sh = O.sigmas(10, shift)
+        assert sh[0] == 1.0 and sh[-1] == 0.0 and np.all(sh[1:-1] > base[1:-1])
+    assert np.all(O.sigmas(10, 0.5)[1:-1] < base[1:-1])
+
+
 def test_euler_constant_velocity():
     """Constant v: x_N = x_0 + (sigma_N - sigma_0) v = x_0 - v exactly."""
     rng = np.random.default_rng(13)
@@ -347,6 +402,32 @@ def test_hv_dual_with_shared_weights_equals_cog_block():
     ref = O.cog_block(x, np.concatenate([m6, m6]), wc, cfg.grid, cfg.heads, 5)
     yt, yv = O.hv_dual_block(x[:5], x[5:], m6, m6, wd, cfg.grid, cfg.heads)
     np.testing.assert_allclose(np.concatenate([yt, yv]), ref, atol=1e-12)
+
+
+def test_hv_dual_streams_are_interchangeable_without_rope():
+    """Without RoPE the dual-stream block treats its two streams alike.
+    Swapping the text and video inputs, modulations and per-stream weights
+    swaps the outputs, since joint attention does not depend on the order of
+    its keys.  A stream that reaches for the other stream's weights, gate or
+    modulation breaks the symmetry."""
+    cfg = _small("hv", n_text=5, dtype="fp32")
+    w = S.block_weights(cfg, 0, 0, block_type="hv_dual")
+    ws = {}
+    for k, v in w.items():
+        if k.startswith("txt."):
+            ws["vid." + k[4:]] = v
+        elif k.startswith("vid."):
+            ws["txt." + k[4:]] = v
+        else:
+            ws[k] = v
+    rng = np.random.default_rng(23)
+    mt, mv = 0.3 * rng.normal(size=6 * cfg.d), 0.3 * rng.normal(size=6 * cfg.d)
+    xt, xv = S.hidden(cfg, 5, tag="txt"), S.hidden(cfg, 9, tag="vid")
+    yt, yv = O.hv_dual_block(xt, xv, mt, mv, w, cfg.grid, cfg.heads, rope=False)
+    yv2, yt2 = O.hv_dual_block(xv, xt, mv, mt, ws, cfg.grid, cfg.heads, rope=False)
+    np.testing.assert_allclose(yt2, yt, atol=1e-12)
+    np.testing.assert_allclose(yv2, yv, atol=1e-12)
+    assert np.abs(yt - xt).max() > 1e-3 and np.abs(yv - xv).max() > 1e-3
 
 
 def test_cog_text_modulation_only_touches_text_rows():
