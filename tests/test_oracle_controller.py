@@ -209,6 +209,85 @@ def test_loop_signals_are_consecutive_temni_drifts(toy):
     assert all(rec.signal > 0 for rec in r.records[1:])
 
 
+def test_teacache_signals_follow_consecutive_steps_through_skips(toy):
+    """TeaCache's signal compares the TEMNIs of consecutive steps, whether the
+    earlier one was computed or reused (Sec. 2).  With every non-warmup step
+    reused the trajectory can be replayed by hand (final layer on
+    H_in + R_0), and each recorded s_t must equal rel_l1(TEMNI_{t-1},
+    TEMNI_t) along it; comparing against the last computed step's TEMNI
+    instead fails from step 2 on."""
+    cfg, w, lat = toy
+    r = O.denoise_loop(cfg, w, lat, None, tau_low=1e9, tau_high=1e9)
+    assert r.computed == [True] + [False] * (cfg.steps - 1)
+    sig = O.sigmas(cfg.steps)
+    x = lat.astype(np.float64)
+    si = O.step_inputs(cfg, w, x, 1000.0 * sig[0])
+    R0 = O.block_stack(cfg, w, si.h_in, si.mods, None) - si.h_in
+    temni = []
+    for i in range(cfg.steps):
+        si = O.step_inputs(cfg, w, x, 1000.0 * sig[i])
+        temni.append(O.block0_temni(cfg, w, si.h_in, si.temb))
+        x = x + (sig[i + 1] - sig[i]) * O.final_layer(cfg, w, si.h_in + R0, si.final_mod)
+    for i in range(1, cfg.steps):
+        assert r.records[i].signal == pytest.approx(O.rel_l1(temni[i - 1], temni[i]), rel=1e-12)
+
+
+def test_easycache_state_through_a_skip_then_compute():
+    """EasyCache's rate k and its previous input and output are those of the
+    step before, whether that step was computed or reused (R9: k = output
+    change over input change between steps c-1 and c, refreshed on every
+    computed step).  Forced decisions compute, compute (warm-up), skip,
+    compute, skip, skip; the hand replay below keeps x_{t-1}, v_{t-1} of the
+    previous step and refreshes k at step 3 against the reused step 2."""
+    cfg = S.get_config("toy", steps=6, method="easycache", tau_low=0.02, tau_high=0.04)
+    w = S.model_weights(cfg, 3)
+    lat = S.latent(cfg, 3)
+    forced = [None, None, False, True, False, False]
+    r = O.denoise_loop(cfg, w, lat, None, forced=forced)
+    assert r.computed == [True, True, False, True, False, False]
+    sig = O.sigmas(cfg.steps)
+    x = lat.astype(np.float64)
+    xs, vs, s_hand = [], [], {}
+    k = x_c = v_c = None
+    for i in range(cfg.steps):
+        if i >= 2:
+            dx = np.abs(x - xs[-1]).mean()
+            s_hand[i] = k * dx / np.abs(vs[-1]).mean()
+        if r.computed[i]:
+            v = O.denoiser(cfg, w, x, 1000.0 * sig[i], None)
+            if i >= 1:
+                k = np.abs(v - vs[-1]).mean() / np.abs(x - xs[-1]).mean()
+            x_c, v_c = x, v
+        else:
+            v = x + (v_c - x_c)
+        xs.append(x)
+        vs.append(v)
+        x = x + (sig[i + 1] - sig[i]) * v
+    for i in range(2, cfg.steps):
+        assert r.records[i].signal == pytest.approx(s_hand[i], rel=1e-12), i
+    np.testing.assert_allclose(r.latent, x, rtol=0, atol=1e-12)
+
+
+def test_easycache_rate_with_an_unchanged_input():
+    """The zero-denominator reading of the drift applies to the rate too: an
+    unchanged input with a changed output gives k = inf, with an unchanged
+    output k = 0."""
+    rng = np.random.default_rng(8)
+    x, v1, v2 = rng.normal(size=(3, 5)), rng.normal(size=(3, 5)), rng.normal(size=(3, 5))
+    assert math.isinf(O.easycache_rate(x, x, v1, v2))
+    assert O.easycache_rate(x, x, v1, v1) == 0.0
+
+
+def test_force_last_leaves_an_explicit_decision_alone(toy):
+    """A decision forced for the last step wins over force_last: an explicit
+    skip stays a skip."""
+    cfg, w, lat = toy
+    forced = [None] * (cfg.steps - 1) + [False]
+    r = O.denoise_loop(cfg, w, lat, None, tau_low=-1.0, tau_high=-1.0, forced=forced, force_last=True)
+    assert r.computed == [True] * (cfg.steps - 1) + [False]
+    assert r.records[-1].forced
+
+
 def test_easycache_affine_model_is_exact():
     """EasyCache (Sec. 2): if the model's output is its input plus a constant
     offset, k = 1 and the reuse x_t + (v_c - x_c) is exact, so any decision
@@ -274,6 +353,34 @@ def test_dicache_single_cached_step_reuses_deep_part():
     p, d, pt = rng.normal(size=(3, 4)), rng.normal(size=(3, 4)), rng.normal(size=(3, 4))
     assert O.dicache_gamma(pt, p, p) == 0.0
     np.testing.assert_allclose(O.dicache_reuse(pt, p, p, d, d), pt + d, atol=0)
+
+
+def test_dicache_reuses_along_the_last_two_computed_steps():
+    """After computed steps 0, 1 and 2 a skipped step extrapolates from the
+    probe and deep parts of steps 2 (latest) and 1: the hand replay below
+    keeps those two, so keeping only the latest (gamma = 0) or the first
+    computed step fails."""
+    cfg = S.get_config("toy", steps=5)
+    w = S.model_weights(cfg, 12)
+    lat = S.latent(cfg, 12)
+    forced = [None, True, True, False, False]
+    r = O.denoise_loop(cfg, w, lat, None, method="dicache", probe_blocks=1, forced=forced)
+    assert r.computed == [True, True, True, False, False]
+    sig = O.sigmas(cfg.steps)
+    x = lat.astype(np.float64)
+    hist = []  # (probe, deep part) of computed steps, latest last
+    for i in range(cfg.steps):
+        si = O.step_inputs(cfg, w, x, 1000.0 * sig[i])
+        probe = O.run_block_range(cfg, w, si.h_in, si.mods, None, 0, 1)
+        if r.computed[i]:
+            h = O.run_block_range(cfg, w, probe, si.mods, None, 1, cfg.n_blocks)
+            hist.append((probe, h - probe))
+        else:
+            (p2, d2), (p1, d1) = hist[-2], hist[-1]
+            g = np.abs(probe - p1).sum() / np.abs(p1 - p2).sum()
+            h = probe + d1 + g * (d1 - d2)
+        x = x + (sig[i + 1] - sig[i]) * O.final_layer(cfg, w, h, si.final_mod)
+    np.testing.assert_allclose(r.latent, x, rtol=0, atol=1e-12)
 
 
 def test_dicache_full_depth_probe_is_uncached():

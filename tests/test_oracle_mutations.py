@@ -154,6 +154,32 @@ MUTANTS = [
     ("dual-stream video FFN input on the text modulation",
      [("    hv = modulate(layer_norm(yv, eps), mv[3], mv[4])", "    hv = modulate(layer_norm(yv, eps), mt[3], mt[4])")],
      [P], "interchangeable"),
+    ("TeaCache signal against the last computed step's TEMNI",
+     [("            self.temni_prev = temni\n            if compute:\n",
+       "            if compute:\n                self.temni_prev = temni\n")], [C], "consecutive_steps_through"),
+    ("EasyCache rate against the last computed step",
+     [("self.k_rate = easycache_rate(x, self.x_prev, v, self.v_prev)",
+       "self.k_rate = easycache_rate(x, self.x_c, v, self.v_c)")], [C], "skip_then_compute"),
+    ("EasyCache previous input and output kept from computed steps only",
+     [("                v = easycache_reuse(x, self.x_c, self.v_c)\n            self.x_prev, self.v_prev = x, v",
+       "                v = easycache_reuse(x, self.x_c, self.v_c)\n            if compute:\n"
+       "                self.x_prev, self.v_prev = x, v")], [C], "skip_then_compute"),
+    ("EasyCache rate 0 for an unchanged input",
+     [("        return 0.0 if dv == 0.0 else math.inf\n    return dv / dx", "        return 0.0\n    return dv / dx")],
+     [C], "unchanged_input"),
+    ("force_last overrides an explicit skip",
+     [("        if force_last and i == n_steps - 1 and f is None:", "        if force_last and i == n_steps - 1:")],
+     [C], "explicit_decision"),
+    ("DiCache keeps only the latest computed step",
+     [("                    self.p_c2, self.d_c2 = self.p_c1, self.d_c1", "                    self.p_c2, self.d_c2 = probe, d_new")],
+     [C], "last_two_computed"),
+    ("joint stack with the video rows first",
+     [("    return np.concatenate([np.asarray(ctx, F64), np.asarray(h_in, F64)], axis=0)",
+       "    return np.concatenate([np.asarray(h_in, F64), np.asarray(ctx, F64)], axis=0)")],
+     [P], "identity_blocks_returns"),
+    ("guided branches share one branch state",
+     [("    bu = SamplerBranch(cfg, w, text_uncond, tau_low, tau_high, delta, warmup, method, probe_blocks, signal_poly)",
+       "    bu = bc")], [G], "branch_state"),
     ("guidance extrapolates from the conditional branch",
      [("return v_uncond + scale * (v_cond - v_uncond)", "return v_cond + scale * (v_uncond - v_cond)")],
      [G], "guidance or unit_and_zero"),

@@ -404,6 +404,35 @@ def test_hv_dual_with_shared_weights_equals_cog_block():
     np.testing.assert_allclose(np.concatenate([yt, yv]), ref, atol=1e-12)
 
 
+@pytest.mark.parametrize("kind", ["cog", "hv"])
+def test_joint_stack_of_identity_blocks_returns_the_video_input(kind):
+    """Joint sequences hold the text rows first.  With every gate zero each
+    block is the identity, so the stack must hand back the video tokens it
+    was given; a stack that put the video first would return a shifted mix
+    of video and text rows."""
+    cfg = _small(kind, n_text=5, dtype="fp32", n_blocks=1, **({"n_single": 1} if kind == "hv" else {}))
+    w = S.model_weights(cfg, 2)
+    h_in = S.hidden(cfg, cfg.n_video, tag="vid")
+    ctx = S.hidden(cfg, 5, tag="txt")
+    d = cfg.d
+    mods = []
+    for wb in w["blocks"]:
+        if "vid.mod" in wb:
+            m = 0.3 * np.ones(6 * d)
+            m[2 * d:3 * d] = m[5 * d:] = 0.0
+            mods.append((m, m))
+        elif kind == "cog":
+            m = 0.3 * np.ones(12 * d)
+            for g in (2, 5, 8, 11):
+                m[g * d:(g + 1) * d] = 0.0
+            mods.append(m)
+        else:
+            m = 0.3 * np.ones(3 * d)
+            m[2 * d:] = 0.0
+            mods.append(m)
+    np.testing.assert_allclose(O.block_stack(cfg, w, h_in, mods, ctx), h_in, atol=1e-12)
+
+
 def test_hv_dual_streams_are_interchangeable_without_rope():
     """Without RoPE the dual-stream block treats its two streams alike.
     Swapping the text and video inputs, modulations and per-stream weights
