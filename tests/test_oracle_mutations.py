@@ -180,6 +180,12 @@ MUTANTS = [
     ("guided branches share one branch state",
      [("    bu = SamplerBranch(cfg, w, text_uncond, tau_low, tau_high, delta, warmup, method, probe_blocks, signal_poly)",
        "    bu = bc")], [G], "branch_state"),
+    ("text projection without its bias",
+     [('        return linear(text, *w["text"])', '        return linear(text, w["text"][0])')], [P], "text_context_closed"),
+    ("dual-stream modulations handed over in swapped order",
+     [('            mods.append((block_modulation(temb, wb["vid.mod"]), block_modulation(temb, wb["txt.mod"])))',
+       '            mods.append((block_modulation(temb, wb["txt.mod"]), block_modulation(temb, wb["vid.mod"])))')],
+     [P], "reaches_its_own_stream"),
     ("guidance extrapolates from the conditional branch",
      [("return v_uncond + scale * (v_cond - v_uncond)", "return v_cond + scale * (v_uncond - v_cond)")],
      [G], "guidance or unit_and_zero"),

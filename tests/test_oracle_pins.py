@@ -433,6 +433,47 @@ def test_joint_stack_of_identity_blocks_returns_the_video_input(kind):
     np.testing.assert_allclose(O.block_stack(cfg, w, h_in, mods, ctx), h_in, atol=1e-12)
 
 
+def test_text_context_closed_forms():
+    """Wan projects the text once (Linear d_text -> d): a zero weight leaves
+    its bias on every text token.  The joint models take the text tokens as
+    given."""
+    cfg = _small("wan", n_text=5, d_text=12, dtype="fp32")
+    w = S.model_weights(cfg, 0, blocks=False)
+    text = S.text(cfg, 0)
+    b = 0.1 * np.arange(cfg.d, dtype=float)
+    ctx = O.text_context(cfg, dict(w, text=(np.zeros((cfg.d, 12)), b)), text)
+    np.testing.assert_array_equal(ctx, np.broadcast_to(b, (5, cfg.d)))
+    cog = _small("cog", n_text=5, dtype="fp32")
+    t = S.hidden(cog, 5, tag="txt")
+    np.testing.assert_array_equal(O.text_context(cog, {}, t), t)
+
+
+def test_dual_stream_step_modulation_reaches_its_own_stream():
+    """A dual-stream block whose video gates are zero leaves the video tokens
+    unchanged, whatever the text stream's modulation: an HV step's block
+    stack must return its video input when only the video modulation's gate
+    rows are zeroed, and must not when only the text's are."""
+    cfg = _small("hv", n_text=5, dtype="fp32", n_blocks=1)
+    w = S.model_weights(cfg, 4)
+    lat = S.latent(cfg, 4)
+    text = S.hidden(cfg, 5, tag="txt")
+    d = cfg.d
+
+    def zero_gates(mod):
+        W, b = (np.array(a, dtype=float) for a in mod)
+        for g in (2, 5):
+            W[g * d:(g + 1) * d] = 0.0
+            b[g * d:(g + 1) * d] = 0.0
+        return W, b
+
+    for stream, identity in (("vid.mod", True), ("txt.mod", False)):
+        blocks = [dict(w["blocks"][0], **{stream: zero_gates(w["blocks"][0][stream])})]
+        wz = dict(w, blocks=blocks)
+        si = O.step_inputs(cfg, wz, lat, 700.0)
+        out = O.block_stack(cfg, wz, si.h_in, si.mods, text)
+        assert np.allclose(out, si.h_in, atol=1e-12) == identity, stream
+
+
 def test_hv_dual_streams_are_interchangeable_without_rope():
     """Without RoPE the dual-stream block treats its two streams alike.
     Swapping the text and video inputs, modulations and per-stream weights
