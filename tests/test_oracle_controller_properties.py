@@ -6,9 +6,11 @@ signals alone (|s_t - s_prev| against delta), so Algorithm 1 is a greedy
 reset rule under a per-step threshold tau_t in [tau_low, tau_high]:
 accumulate, skip while the sum stays within tau_t, otherwise compute and
 reset.  A greedy rule under pointwise larger thresholds never computes more
-often.  By induction, its running sum after any step is at most the other
-rule's whenever both have computed equally often.  Hence the compute counts
-sit between those of the fixed thresholds.  The other properties are special
+often: by induction on k, its k-th compute never comes before the other
+rule's k-th compute.  Once the other rule has restarted its sum no later,
+that sum covers at least as many non-negative signals, against a threshold
+no larger.  Hence the compute counts sit between those of the fixed
+thresholds.  The other properties are special
 cases of the rule: equal thresholds, a negative delta, zero signals, and a
 power-of-two rescaling of every quantity (exact in binary floating point).
 """
