@@ -35,8 +35,11 @@ METRIC = "DiT steps/s and attention TFLOP/s (% bf16 peak), Wan-1.3B-shaped 480p"
 UNIT = "steps/s"
 WORKLOAD = ("Wan-2.1-1.3B-shaped 480p step: 30 blocks, d=1536, 12 heads x 128, FFN 8960, "
             "32760 video tokens (21x30x52, 3D RoPE), cross-attention to 512 text tokens (4096 -> 1536)")
-CPU_SAMPLE_ROWS = 4096
-REF_SAMPLE_ROWS = 2048
+# Query rows of the oracle sample, the same for the GPU arm's cpu_baseline and
+# for the reference arm (about 7 s of fp64 numpy work per sample on 16 cores).
+SAMPLE_ROWS = 2048
+MICRO_T = (32760, 67320, 118800)  # drift micro-benchmark rows (x 3072 bf16)
+MICRO_SIGMA = 1e-2
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, ncu captures of
 # a self-attention call (main launch, split tail launch and merge) and a
@@ -203,30 +206,184 @@ def _cores() -> int:
         return os.cpu_count() or 1
 
 
+def _config(seq_len: int) -> dict:
+    """The workload description both arms print (identical keys and values)."""
+    return {"workload": WORKLOAD, "global_batch": 1, "seq_len": seq_len, "parallelism": "replicas",
+            "schedule": "every step computed (tau_low = tau_high = -1); drift and decision still run",
+            "l2": "no flush: per-step working set (3.4 GB of bf16 weights read once per step, >0.5 GB "
+                  "activations) exceeds the 129 MB L2"}
+
+
+def baseline_record(sample: "OracleSample", seconds: list[float]) -> dict:
+    """cpu_baseline object of a timed oracle sample: the step rate is the
+    sample's FLOP-scaled rate (extrapolated, not timed as a whole step)."""
+    mean = sum(seconds) / len(seconds)
+    return {"value": sample.steps_per_s(mean), "unit": UNIT, "cores": _cores(), "kind": "oracle",
+            "sample": sample.describe(), "extrapolated_from_rows": sample.R,
+            "sample_seconds": mean, "samples_timed": len(seconds),
+            "scaled_by": "algorithmic FLOPs of one 30-block step / FLOPs of the sample"}
+
+
 def run_reference(args) -> None:
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    s = OracleSample(REF_SAMPLE_ROWS)
+    s = OracleSample(SAMPLE_ROWS)
     for _ in range(args.warmup):
         s.run()
     times = [s.run() for _ in range(args.steps)]
-    total = sum(times)
-    value = s.steps_per_s(total / len(times))
+    base = baseline_record(s, times)
+    value = base["value"]
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / value,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": WORKLOAD, "global_batch": 1, "seq_len": 32760,
-                                            "parallelism": "replicas"},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": _cores(), "kind": "oracle",
-                             "sample": s.describe()},
-            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "data": "synthetic (random N(0,0.02) weights, N(0,1) latent and text)",
+            "config": _config(32760),
+            "cpu_baseline": base,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "note": "each timed step is one oracle sample of %d query rows (%.1f s); ms_per_step is the "
+                    "FLOP-scaled time of a whole 30-block step, not a timed step" % (s.R, base["sample_seconds"])}
     print(json.dumps(line), flush=True)
 
 
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+
+def _launch_ms(fn, iters: int, flush=None) -> float:
+    """Mean device time of one call of fn: CUDA events around each call on the
+    current stream, with `flush` (an untimed write larger than L2) between calls."""
+    import torch
+
+    st = torch.cuda.current_stream()
+    total = 0.0
+    for _ in range(iters):
+        if flush is not None:
+            flush.add_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        fn()
+        e1.record(st)
+        e1.synchronize()
+        total += e0.elapsed_time(e1)
+    return total / iters
+
+
+def micro_bench(acid, dev, peaks: dict, iters: int = 5) -> dict:
+    """Drift reduction, stand-alone cache apply and the fused drift + apply on
+    [T, 3072] bf16 (prev ~ N(0,1), cur = prev + 0.01 z), L2 flushed between
+    launches.  Algorithmic bytes per element: drift 4 (reads prev, cur), apply 6
+    (reads x, residual, writes out), fused 8 (reads prev, cur, residual, writes out)."""
+    import torch
+
+    gen = torch.Generator(device=dev).manual_seed(7)
+    flush = torch.zeros(64 << 20, dtype=torch.float32, device=dev)  # 256 MB > 129 MB L2
+    hbm = peaks["hbm_gbs"]
+    out = {"d": 3072, "sigma": MICRO_SIGMA, "l2": "flushed between launches (256 MB write)", "rows": {}}
+    worst = {"drift": 1.0, "apply": 1.0, "fused": 1.0}
+    for T in MICRO_T:
+        n = T * 3072
+        p = torch.randn(n, device=dev, generator=gen).to(torch.bfloat16)
+        c = (p.float() + MICRO_SIGMA * torch.randn(n, device=dev, generator=gen)).to(torch.bfloat16)
+        r = torch.randn(n, device=dev, generator=gen).to(torch.bfloat16)
+        o = torch.empty_like(p)
+        ws = torch.empty(acid.drift_workspace_size(n), dtype=torch.uint8, device=dev)
+        rel = torch.empty(1, dtype=torch.float64, device=dev)
+        sums = torch.empty(2, dtype=torch.float64, device=dev)
+        runs = {
+            "drift": (lambda: acid.acid_drift_signal(p, c, out_rel=rel, out_sums=sums, workspace=ws), 4.0,
+                      "drift_partials_kernel + drift_final_kernel"),
+            "apply": (lambda: acid.acid_cache_apply(c, r, out=o), 6.0, "add_vec_kernel"),
+            "fused": (lambda: acid.acid_drift_apply(p, c, r, out=o, out_rel=rel, out_sums=sums, workspace=ws), 8.0,
+                      "drift_partials_kernel<apply> + drift_final_kernel"),
+        }
+        row = {}
+        for name, (fn, bpe, kern) in runs.items():
+            fn()
+            ms = _launch_ms(fn, iters, flush)
+            gbs = bpe * n / ms / 1e6
+            row[name] = {"ms": ms, "gbs": gbs, "frac_of_hbm": gbs / hbm, "bytes_per_elem": bpe, "kernel": kern}
+            worst[name] = min(worst[name], gbs / hbm)
+        torch.cuda.synchronize()
+        row["rel_l1"] = rel.item()
+        out["rows"][str(T)] = row
+        del p, c, r, o, ws
+    out["min_frac_of_hbm"] = worst
+    out["hbm_peak"] = hbm
+    torch.cuda.empty_cache()
+    return out
+
+
+def block_bench(acid, dev, peaks: dict, iters: int = 3) -> dict:
+    """One block of each other workload at full length (random N(0, 0.02)
+    weights of that block, N(0, 1) input): block ms, and the attention and
+    GEMM rates inside it from the library's per-launch CUDA events."""
+    import torch
+
+    import acid_synth as S
+
+    res = {}
+    for wl, bt in (("cog", "cog"), ("hv", "hv_dual"), ("hv", "hv_single")):
+        cfg = S.get_config(wl)
+        w = S.block_weights(cfg, 0, seed=0, block_type=bt)
+        blk = acid.DeviceBlock.upload(w, bt, torch.bfloat16, dev)
+        del w
+        rows = cfg.n_video + cfg.n_text
+        desc = acid.block_desc(cfg, bt)
+        gen = torch.Generator(device=dev).manual_seed(11)
+        temb = torch.from_numpy(S.temb_vector(cfg, 0)).to(dev)
+        x0 = torch.randn(rows, cfg.d, device=dev, generator=gen).to(torch.bfloat16)
+        x = x0.clone()
+        ws = torch.empty(acid.block_workspace_size(desc) + 1024, dtype=torch.uint8, device=dev)
+
+        def run():
+            acid.acid_dit_block_forward(desc, x, temb, blk, workspace=ws)
+
+        for _ in range(2):
+            x.copy_(x0)
+            run()
+        torch.cuda.synchronize()
+        ms_total = 0.0
+        acid.profile_enable(True)
+        for _ in range(iters):
+            x.copy_(x0)
+            ms_total += _launch_ms(run, 1)
+        a_n, a_ms, a_flop = acid.profile_read(acid.PROF_ATTENTION)
+        l_n, l_ms, l_flop = acid.profile_read(acid.PROF_LINEAR)
+        acid.profile_enable(False)
+        acid.check_device_error()
+        att = a_flop / (a_ms / 1000.0) / 1e12 if a_ms > 0 else None
+        lin = l_flop / (l_ms / 1000.0) / 1e12 if l_ms > 0 else None
+        res[f"{wl}/{bt}"] = {
+            "rows": rows, "d": cfg.d, "heads": cfg.heads, "head_dim": cfg.head_dim, "block_ms": ms_total / iters,
+            "attention_tflops": att, "attention_frac_of_burst_peak": att / peaks["bf16_tflops"] if att else None,
+            "attention_ms": a_ms / iters, "linear_tflops": lin, "linear_ms": l_ms / iters,
+            "step_ms_estimate": ms_total / iters * (cfg.n_blocks if bt != "hv_single" else cfg.n_single),
+        }
+        del blk, x, x0, ws
+        torch.cuda.empty_cache()
+    res["note"] = ("one block timed alone, CUDA events; step_ms_estimate = block_ms x blocks of that kind; "
+                   "working sets exceed L2 (no flush)")
+    return res
+
+
+def toy_bench(acid, dev, steps: int = 10) -> dict:
+    """The fp32 toy DiT (2 blocks, d 256, 256 tokens): every step of a 10-step
+    generation computed, device time per step."""
+    import torch
+
+    import acid_synth as S
+
+    cfg = S.get_config("toy")
+    model = acid.DeviceModel(cfg, S.model_weights(cfg, 0), dev)
+    lat0 = torch.from_numpy(S.latent(cfg, 0)).to(dev)
+    c, keep = acid.loop_cfg(cfg, n_steps=steps, tau_low=-1.0, tau_high=-1.0)
+    loop = acid.Loop(model, c, None, dev)
+    lat = lat0.clone()
+    loop.step(lat, log=False)
+    ms = _launch_ms(lambda: [loop.step(lat, log=False) for _ in range(steps - 1)], 1) / (steps - 1)
+    return {"step_ms": ms, "steps_per_s": 1000.0 / ms, "dtype": "f32", "tokens": cfg.n_video, "blocks": cfg.n_blocks}
+
 
 def run_ours(args) -> None:
     import numpy as np
@@ -341,9 +498,7 @@ def run_ours(args) -> None:
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic (random N(0,0.02) weights, N(0,1) latent and text)",
-        "config": {"workload": WORKLOAD, "global_batch": 1, "seq_len": cfg.n_video, "parallelism": "replicas",
-                   "schedule": "every step computed (tau_low = tau_high = -1); drift and decision still run",
-                   "l2": "no flush: per-step working set (3.4 GB of bf16 weights read once per step, >0.5 GB activations) exceeds the 129 MB L2"},
+        "config": _config(cfg.n_video),
         "roofline": {"bound": "tensor", "kernel": "attn_tc_kernel<128> (self) + attn_persist_kernel<128> (cross attention)",
                      "achieved": att_tflops, "peak": peak, "unit": "TFLOP/s", "frac": att_tflops / peak,
                      "peak_source": f"bf16_tflops_sustained, {src}", "traffic": _attn_traffic(),
@@ -367,11 +522,13 @@ def run_ours(args) -> None:
         "gpu_launches": launches,
         "clocks": clk.summary(),
     }
+    if not args.no_extras:
+        line["micro"] = micro_bench(acid, dev, peaks)
+        line["blocks"] = block_bench(acid, dev, peaks)
+        line["toy"] = toy_bench(acid, dev)
     if not args.no_cpu_baseline and world == 1:
-        s = OracleSample(CPU_SAMPLE_ROWS)
-        secs = s.run()
-        line["cpu_baseline"] = {"value": s.steps_per_s(secs), "unit": UNIT, "cores": _cores(), "kind": "oracle",
-                                "sample": s.describe() + f"; {secs:.1f} s"}
+        s = OracleSample(SAMPLE_ROWS)
+        line["cpu_baseline"] = baseline_record(s, [s.run()])
     print(json.dumps(line), flush=True)
 
 
@@ -382,6 +539,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the per-workload blocks, the drift micro-benchmark and the toy step")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)  # at least three untimed warm-up steps
     if args.impl == "reference":

@@ -143,14 +143,19 @@ acid_status acid_cache_apply(const void* x, const void* cached_residual, void* o
  * fully reserved by another allocator.  The paper has no counterpart: this is
  * a deployment variant of the drift reduction above, with the same result.
  *   Arguments and outputs as acid_drift_signal (device or host outputs).
- *   n          0 <= n <= 2^33; larger n fails with ACID_ERR_UNSUPPORTED.
+ *   n          0 <= n <= 2^31; larger n fails with ACID_ERR_UNSUPPORTED (the
+ *              limit keeps the worst-case fp32 rounding of the per-thread sums
+ *              inside the 1e-3 drift tolerance).
  * Scratch: a 16 KiB array in the library's device memory, held by every GPU
  * that loads the library until the process exits.  No cudaMalloc, cudaFree
  * or allocating library call is made.  The first call on each device looks
  * up the array's device address (cudaGetSymbolAddress); make that first call
- * outside any stream capture.  All calls share the array and it keeps the
- * last call's contents: calls that overlap on the GPU (different streams
- * without ordering) race and give undefined results. */
+ * outside any stream capture.  The lookup is repeated when the device's
+ * context has been replaced (cudaDeviceReset reloads the library's device
+ * code at a new address); the first call after a reset is again a set-up
+ * call.  All calls share the array and it keeps the last call's contents:
+ * calls that overlap on the GPU (different streams without ordering) race and
+ * give undefined results. */
 acid_status acid_drift_signal_noalloc(const void* prev, const void* cur, int64_t n, int32_t dtype,
                                       double* out_rel_l1, double* out_sums, acid_stream_t stream);
 

@@ -303,7 +303,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint64_t* empty = full + C::STAGES;
   uint64_t* acc_full = empty + C::STAGES;  // [2]
   uint64_t* acc_empty = acc_full + 2;      // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  uint64_t* drain = acc_empty + 2;         // failure path: the MMAs issued so far have completed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int num_kb = (g.K + BK - 1) / BK;
@@ -321,6 +322,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 32 * kEpiWarps);
     }
+    mbar_init(drain, 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -343,6 +345,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           tma_load_2d(sB + s * C::B_BYTES, &tmB, &full[s], kb * BK, n_tile * BN);
         }
       }
+      // After a wait ran out: the loads of the last STAGES issues may still be
+      // in flight; wait (bounded) until they have landed, so that no TMA
+      // writes into this CTA's shared memory after it exits.  Earlier issues
+      // were consumed by the MMA thread before their stage was refilled.
+      if (!ok)
+        for (int j = std::max(0, it - C::STAGES); j < it; ++j) mbar_wait(&full[j % C::STAGES], (j / C::STAGES) & 1);
     }
   } else if (warp == 1) {
     if (lane == 0) {  // MMA issuer
@@ -369,6 +377,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           mma_commit(&empty[s]);
         }
         if (ok) mma_commit(&acc_full[b]);
+      }
+      // After a wait ran out: let the MMAs already issued finish (bounded)
+      // before the accumulator's tensor memory is freed below.
+      if (!ok) {
+        mma_commit(drain);
+        mbar_wait(drain, 0);
       }
     }
   } else {  // epilogue: warps 2..9; lane quarter = warp % 4, column half = (warp - 2) / 4

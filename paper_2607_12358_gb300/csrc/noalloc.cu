@@ -8,6 +8,8 @@
 // three results) lives in the file-scope array below instead of a
 // caller-provided workspace.  Every GPU that loads this library holds the
 // array until the process exits.
+#include <cudaTypedefs.h>
+
 #include <mutex>
 #include <string>
 
@@ -21,31 +23,68 @@ bool is_device_pointer(const void* p);
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = 16 * 1024;
-// Largest element count accepted: the grid is capped at a fixed number of
-// thread blocks, so each thread's fp32 partial sums cover at most about 55,000
-// values at this size, which keeps their rounding far below the 1e-3 drift
-// tolerance.
-constexpr int64_t kNoAllocMaxElems = int64_t(1) << 33;
+// Largest element count accepted.  The reduction runs a fixed grid of 608
+// blocks of 256 threads, and each thread sums |cur - prev| and |prev| into
+// two fp32 accumulators each, so at n = 2^31 an accumulator adds at most
+// 2^31 / (608 * 256 * 2) < 6,900 terms.  Summing non-negative terms one by one
+// in fp32 has a relative error of at most (terms - 1) * 2^-24 < 4.2e-4, and
+// the fp64 stages after it add nothing at that scale, so the ratio of the two
+// sums stays within about 8.4e-4 of exact even in the worst case: inside the
+// 1e-3 drift tolerance.  (The expected error, which grows with the square
+// root of the term count, is far smaller.)
+constexpr int64_t kNoAllocMaxElems = int64_t(1) << 31;
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 std::mutex g_mu;
-void* g_scratch_addr[kMaxDevices] = {};
+struct ScratchSlot {
+  CUcontext ctx;  // context the address belongs to
+  void* addr;
+};
+ScratchSlot g_slot[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device, looked up once
-// per device (host code cannot use the symbol itself as a device pointer).
+// cuCtxGetCurrent through the runtime's driver entry-point query (the library
+// does not link the driver API).
+PFN_cuCtxGetCurrent_v4000 ctx_get_current() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+  });
+  return fn;
+}
+
+// Device address of the scratch array in the current device's context (host
+// code cannot use the symbol itself as a device pointer).  Looked up once per
+// device and looked up again if that device's context has changed since, as
+// after cudaDeviceReset, which reloads the module at a new address.
 acid_status scratch_address(void** out) {
   int dev = 0;
   ACID_CUDA(cudaGetDevice(&dev));
   ACID_REQUIRE(dev >= 0 && dev < kMaxDevices, ACID_ERR_UNSUPPORTED, "drift_noalloc: device index too large");
+  auto get_ctx = ctx_get_current();
+  ACID_REQUIRE(get_ctx != nullptr, ACID_ERR_CUDA, "drift_noalloc: cuCtxGetCurrent entry point unavailable");
   std::lock_guard<std::mutex> lk(g_mu);
-  if (g_scratch_addr[dev] == nullptr) {
-    void* p = nullptr;
-    ACID_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch));
-    g_scratch_addr[dev] = p;
+  ScratchSlot& sl = g_slot[dev];
+  CUcontext ctx = nullptr;
+  if (sl.addr != nullptr && get_ctx(&ctx) == CUDA_SUCCESS && ctx == sl.ctx) {
+    *out = sl.addr;
+    return ACID_OK;
   }
-  *out = g_scratch_addr[dev];
+  // first call on this device, or its context was replaced: the lookup also
+  // makes the device's primary context current, so the context is read after it
+  void* p = nullptr;
+  ACID_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch));
+  ctx = nullptr;
+  ACID_REQUIRE(get_ctx(&ctx) == CUDA_SUCCESS && ctx != nullptr, ACID_ERR_CUDA, "drift_noalloc: no current context");
+  sl.ctx = ctx;
+  sl.addr = p;
+  *out = p;
   return ACID_OK;
 }
 

@@ -1,7 +1,8 @@
 """acid_drift_signal_noalloc: the drift reduction for callers that cannot
 allocate device memory (not even a workspace), checked through the C ABI
 against acid_drift_signal, the entry point that takes a caller-provided
-workspace.  Two calls in a row, so a stale scratch array would show.
+workspace, and against the fp64 CPU oracle.  Two calls in a row, so a stale
+scratch array would show.
 
 This file is collected last so that a run stopping at the first failure has
 already run every other test; it also passes on its own in a fresh process.
@@ -13,6 +14,7 @@ import numpy as np
 import pytest
 
 import acid_synth as S
+import oracle as O
 
 pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
@@ -69,6 +71,11 @@ def test_noalloc_matches_workspace_entry_point_twice(lib):
         rel, sums = _noalloc_call(A, tp, tc, dt)
         assert abs(rel - ref_rel) <= DRIFT_RTOL * ref_rel
         np.testing.assert_allclose(sums, ref_sums, rtol=DRIFT_RTOL)
+        # the same inputs in the fp64 oracle (the device values, upcast)
+        p64, c64 = tp.double().cpu().numpy(), tc.double().cpu().numpy()
+        orel = O.rel_l1(p64, c64)
+        assert abs(rel - orel) <= DRIFT_RTOL * orel, (rel, orel)
+        np.testing.assert_allclose(sums, [np.abs(c64 - p64).sum(), np.abs(p64).sum()], rtol=DRIFT_RTOL)
         hrel, hsums = _noalloc_call(A, tp, tc, dt, host=True)
         assert abs(hrel - ref_rel) <= DRIFT_RTOL * ref_rel
         np.testing.assert_allclose(hsums, ref_sums, rtol=DRIFT_RTOL)
@@ -78,7 +85,7 @@ def test_noalloc_rejects_sizes_beyond_maximum(lib):
     A = lib
     out = torch.zeros(1, dtype=torch.float64, device=DEV)
     x = torch.zeros(16, dtype=torch.bfloat16, device=DEV)
-    st = A.load().acid_drift_signal_noalloc(x.data_ptr(), x.data_ptr(), (1 << 33) + 1, A.ACID_BF16,
+    st = A.load().acid_drift_signal_noalloc(x.data_ptr(), x.data_ptr(), (1 << 31) + 1, A.ACID_BF16,
                                             out.data_ptr(), None, None)
     assert st == A.ACID_ERR_UNSUPPORTED
     assert b"maximum" in A.load().acid_last_error()
