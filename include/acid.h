@@ -127,6 +127,27 @@ acid_status acid_drift_signal(const void* prev, const void* cur, int64_t n, int3
                               double* out_rel_l1, double* out_sums, void* workspace,
                               size_t workspace_bytes, acid_stream_t stream);
 
+/* TeaCache signal straight from two consecutive steps' patch embeddings
+ * (Sec. 2, "TeaCache": the drift of the timestep-embedding-modulated noisy
+ * input, TEMNI).  With TEMNI_t = LN(h_t) (1 + scale_t) + shift_t row by row
+ * (LayerNorm without affine parameters, epsilon eps) it returns
+ *     rel_l1 = sum |TEMNI_t - TEMNI_{t-1}| / sum |TEMNI_{t-1}|
+ * as acid_drift_signal does, but forms both TEMNIs in registers in one
+ * read-only pass over the two fp32 inputs (8 bytes read per element, nothing
+ * written but the result): the step loop keeps each step's h and modulation
+ * instead of a stored TEMNI.
+ *   h_prev, h_cur      device fp32 [rows, d], row-major, 16-byte aligned.
+ *   mod_prev, mod_cur  device fp32 [2 d] = {shift[d], scale[d]} of each step.
+ *   rows >= 0; d % 8 == 0 and d <= 3072, else ACID_ERR_UNSUPPORTED.
+ *   out_rel_l1, out_sums   as acid_drift_signal (device or host; host makes
+ *                          the call synchronous).
+ *   workspace  device, >= acid_drift_workspace_size(rows * d) bytes,
+ *              16-byte aligned.
+ * rows = 0 gives 0 (and zero sums). */
+acid_status acid_temni_drift(const float* h_prev, const float* h_cur, const float* mod_prev, const float* mod_cur,
+                             int64_t rows, int32_t d, float eps, double* out_rel_l1, double* out_sums,
+                             void* workspace, size_t workspace_bytes, acid_stream_t stream);
+
 /* Cached-residual reuse on a skipped step (Sec. 2 "TeaCache": previous output
  * reconstructed with a stored residual; "EasyCache": input plus the offset of
  * the last computed step):  out = x + cached_residual, elementwise, rounded

@@ -84,6 +84,7 @@ _PROTOS = {
     "acid_drift_workspace_size": (C.c_int, [C.c_int64, C.POINTER(C.c_size_t)]),
     "acid_drift_signal": (C.c_int, [_P, _P, C.c_int64, C.c_int32, _P, _P, _P, C.c_size_t, _P]),
     "acid_cache_apply": (C.c_int, [_P, _P, _P, C.c_int64, C.c_int32, _P]),
+    "acid_temni_drift": (C.c_int, [_P, _P, _P, _P, C.c_int64, C.c_int32, C.c_float, _P, _P, _P, C.c_size_t, _P]),
     "acid_drift_signal_noalloc": (C.c_int, [_P, _P, C.c_int64, C.c_int32, _P, _P, _P]),
     "acid_drift_apply": (C.c_int, [_P, _P, _P, _P, C.c_int64, C.c_int32, _P, _P, _P, C.c_size_t, _P]),
     "acid_linear_forward": (C.c_int, [C.c_int32, _P, C.c_int64, C.c_int64, C.c_int32, _P, _P, C.c_int32, _P,

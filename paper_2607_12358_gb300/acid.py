@@ -106,6 +106,28 @@ def acid_drift_signal(prev: torch.Tensor, cur: torch.Tensor, out_rel: torch.Tens
     return out_rel, out_sums
 
 
+def acid_temni_drift(h_prev: torch.Tensor, h_cur: torch.Tensor, mod_prev: torch.Tensor, mod_cur: torch.Tensor,
+                     eps: float = 1e-6, out_rel: torch.Tensor | None = None, out_sums: torch.Tensor | None = None,
+                     workspace: torch.Tensor | None = None, stream=None):
+    """rel_l1(TEMNI_prev, TEMNI_cur) with TEMNI = LN(h) (1 + scale) + shift from
+    fp32 h [rows, d] and mod = [shift | scale] fp32 [2d] of each step."""
+    _need_cuda(h_prev, h_cur, mod_prev, mod_cur)
+    for t in (h_prev, h_cur, mod_prev, mod_cur):
+        if t.dtype != torch.float32 or not t.is_contiguous():
+            raise ValueError("temni_drift inputs must be contiguous fp32")
+    rows, d = h_cur.shape
+    if h_prev.shape != h_cur.shape or mod_prev.numel() != 2 * d or mod_cur.numel() != 2 * d:
+        raise ValueError("temni_drift: shape mismatch")
+    dev = h_cur.device
+    out_rel = torch.empty(1, dtype=torch.float64, device=dev) if out_rel is None else out_rel
+    out_sums = torch.empty(2, dtype=torch.float64, device=dev) if out_sums is None else out_sums
+    ws = torch.empty(drift_workspace_size(rows * d), dtype=torch.uint8, device=dev) if workspace is None else workspace
+    check(load().acid_temni_drift(h_prev.data_ptr(), h_cur.data_ptr(), mod_prev.data_ptr(), mod_cur.data_ptr(), rows,
+                                  d, float(eps), out_rel.data_ptr(), out_sums.data_ptr(), ws.data_ptr(), ws.numel(),
+                                  _stream(stream)))
+    return out_rel, out_sums
+
+
 def acid_cache_apply(x: torch.Tensor, cached_residual: torch.Tensor, out: torch.Tensor | None = None,
                      stream=None) -> torch.Tensor:
     """out = x + cached_residual."""

@@ -169,6 +169,47 @@ extern "C" acid_status acid_drift_workspace_size(int64_t n, size_t* bytes) {
   return ACID_OK;
 }
 
+extern "C" acid_status acid_temni_drift(const float* h_prev, const float* h_cur, const float* mod_prev,
+                                        const float* mod_cur, int64_t rows, int32_t d, float eps, double* out_rel,
+                                        double* out_sums, void* ws, size_t ws_bytes, acid_stream_t stream) {
+  clear_error();
+  cudaStream_t s = (cudaStream_t)stream;
+  ACID_REQUIRE(rows >= 0 && d > 0, ACID_ERR_INVALID_ARG, "temni_drift: rows must be >= 0 and d > 0");
+  ACID_REQUIRE(d % 8 == 0 && d <= 3072, ACID_ERR_UNSUPPORTED, "temni_drift: d must be a multiple of 8, <= 3072");
+  ACID_REQUIRE(out_rel != nullptr, ACID_ERR_INVALID_ARG, "temni_drift: out_rel_l1 is null");
+  ACID_REQUIRE(rows == 0 || (h_prev && h_cur && mod_prev && mod_cur), ACID_ERR_INVALID_ARG, "temni_drift: null input");
+  ACID_REQUIRE(rows == 0 || (aligned(h_prev, 16) && aligned(h_cur, 16) && aligned(mod_prev, 16) && aligned(mod_cur, 16)),
+               ACID_ERR_UNSUPPORTED, "temni_drift: inputs must be 16-byte aligned");
+  ACID_REQUIRE(ws != nullptr && aligned(ws, 16), ACID_ERR_WORKSPACE, "temni_drift: workspace null or not 16-byte aligned");
+  const int64_t n = rows * (int64_t)d;
+  const size_t need = drift_workspace_bytes(n) + 64;
+  ACID_REQUIRE(ws_bytes >= need, ACID_ERR_WORKSPACE,
+               "temni_drift: workspace too small (need " + std::to_string(need) + ")");
+  double* result = reinterpret_cast<double*>(static_cast<uint8_t*>(ws) + drift_workspace_bytes(n));
+  if (rows == 0) {
+    ACID_CUDA(cudaMemsetAsync(result, 0, 3 * sizeof(double), s));
+  } else {
+    ACID_TRY(temni_drift(h_cur, h_prev, mod_cur, mod_prev, nullptr, 1, rows, d, eps, result, ws,
+                         drift_workspace_bytes(n), s));
+  }
+  const bool rel_dev = is_device_pointer(out_rel);
+  const bool sums_dev = out_sums ? is_device_pointer(out_sums) : true;
+  if (rel_dev) ACID_CUDA(cudaMemcpyAsync(out_rel, result, sizeof(double), cudaMemcpyDeviceToDevice, s));
+  if (out_sums && sums_dev)
+    ACID_CUDA(cudaMemcpyAsync(out_sums, result + 1, 2 * sizeof(double), cudaMemcpyDeviceToDevice, s));
+  if (!rel_dev || !sums_dev) {
+    double h[3];
+    ACID_CUDA(cudaMemcpyAsync(h, result, sizeof(h), cudaMemcpyDeviceToHost, s));
+    ACID_CUDA(cudaStreamSynchronize(s));
+    if (!rel_dev) *out_rel = h[0];
+    if (out_sums && !sums_dev) {
+      out_sums[0] = h[1];
+      out_sums[1] = h[2];
+    }
+  }
+  return ACID_OK;
+}
+
 extern "C" acid_status acid_drift_signal(const void* prev, const void* cur, int64_t n, int32_t dtype,
                                          double* out_rel_l1, double* out_sums, void* workspace, size_t workspace_bytes,
                                          acid_stream_t stream) {

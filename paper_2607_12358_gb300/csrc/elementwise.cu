@@ -13,6 +13,16 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kDriftMaxBlocks = 152 * 4;  // one wave of 4 CTAs per SM on GB300
 
+int num_sms_elem() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  }
+  return n;
+}
+
 __device__ __forceinline__ double warp_sum_d(double v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -277,110 +287,176 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
   }
 }
 
-// ------------------------------------------------- fused TEMNI + drift
-// TEMNI_cur = LN(x) (1 + scale) + shift (fp32) and, in the same pass, the
-// sums |TEMNI_cur - TEMNI_prev| and |TEMNI_prev| for the relative-L1 drift.
-// The two TEMNI buffers alternate with the step's parity: cur = tem[step & 1],
-// prev = tem[(step + 1) & 1]; `step` is read from device memory when
-// step_dev is given (graph-launched loops), else step_host is used.  At step
-// 0 there is no previous TEMNI and the sums are zero.  One warp per row
-// (grid-strided), fp64 CTA partials reduced by drift_final_kernel.
-// NV: 8-element vectors per lane (d <= 256 * NV), so that the row held in
-// registers is sized to d.  For rows up to 1536 wide the previous TEMNI row
-// is loaded together with x: a row then costs one DRAM round trip, not two.
-// The arithmetic and its order do not depend on NV.
-template <int NV>
-__global__ void __launch_bounds__(kThreads, 2) ln_mod_drift_kernel(const float* __restrict__ x, float* tem0,
-                                                                   float* tem1, const int* step_dev, int step_host,
-                                                                   int64_t rows, int d,
-                                                                   const float* __restrict__ shift,
-                                                                   const float* __restrict__ scale, float eps,
-                                                                   double2* __restrict__ partials) {
-  constexpr bool kPrevEarly = NV <= 6;
+// ------------------------------------------- TEMNI drift from two H_in rows
+// The sums |TEMNI_t - TEMNI_{t-1}| and |TEMNI_{t-1}| of the TeaCache signal,
+// with TEMNI = LN(H_in) (1 + scale) + shift at each step's own (shift,
+// scale).  Both TEMNI rows are formed in registers from the fp32 patch
+// embeddings H_in_t (xc) and H_in_{t-1} (xp), so the kernel reads 8 bytes per
+// element and writes nothing but one fp64 partial pair per CTA (reduced by
+// drift_final_kernel).
+// One warp per row pair (rows gw, gw + total warps, ...), reductions by warp
+// shuffles only.  Lane 0 of each warp streams the warp's row pairs into its
+// own two-stage shared-memory ring with 1D bulk copies (completion counted on
+// the stage's mbarrier), so the bytes in flight come from shared memory, not
+// registers; the stage is refilled as soon as every lane has read it.  The
+// four modulation vectors (shift and 1 + scale of both steps) are staged once
+// per CTA in shared memory.  Row statistics: mean and variance from sums of
+// (x - K) and (x - K)^2 with K the row's first element, which keeps the
+// fp32 cancellation small (K lies within a few standard deviations of the
+// mean).  HOLD: rows of up to 1536 values stay in registers after one read of
+// the stage (16 per lane), else the stage is read again for the final pass.
+// Step 0 gives zero sums.
+constexpr int kTemniStages = 2;
+constexpr int kTemniMaxWarps = 8;
+
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+template <int NV4, bool HOLD>
+__global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(const float* __restrict__ xc,
+                                                                            const float* __restrict__ xp,
+                                                                            const int* step_dev, int step_host,
+                                                                            int64_t rows, int d,
+                                                                            const float* __restrict__ shc,
+                                                                            const float* __restrict__ scc,
+                                                                            const float* __restrict__ shp,
+                                                                            const float* __restrict__ scp, float eps,
+                                                                            double2* __restrict__ partials) {
+  extern __shared__ __align__(128) uint8_t tsm[];
+  const int nwarps = blockDim.x >> 5;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // four d-long vectors: shift_c, 1 + scale_c, shift_p, 1 + scale_p (separate
+  // arrays, so that a warp's 16-byte reads of one vector are contiguous)
+  float4* mod = reinterpret_cast<float4*>(tsm);
+  float* ring = reinterpret_cast<float*>(tsm + (size_t)16 * d);                       // [warp][stage][2][d]
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)nwarps * kTemniStages * 2 * d);  // [warp][stage]
+  __shared__ double rd[2][kTemniMaxWarps];
   const int step = step_dev ? *step_dev : step_host;
-  float* cur = (step & 1) ? tem1 : tem0;
-  const float* prev = (step & 1) ? tem0 : tem1;
-  const bool has_prev = step > 0;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t gw = (int64_t)blockIdx.x * (kThreads / 32) + warp;
-  const int64_t nw = (int64_t)gridDim.x * (kThreads / 32);
+  for (int i = threadIdx.x; i < d / 4; i += blockDim.x) {
+    const float4 a = reinterpret_cast<const float4*>(shc)[i], b = reinterpret_cast<const float4*>(scc)[i];
+    const float4 c = reinterpret_cast<const float4*>(shp)[i], e = reinterpret_cast<const float4*>(scp)[i];
+    const int q = d / 4;
+    mod[i] = a;
+    mod[q + i] = make_float4(1.f + b.x, 1.f + b.y, 1.f + b.z, 1.f + b.w);
+    mod[2 * q + i] = c;
+    mod[3 * q + i] = make_float4(1.f + e.x, 1.f + e.y, 1.f + e.z, 1.f + e.w);
+  }
+  float* wr = ring + (size_t)warp * kTemniStages * 2 * d;
+  uint64_t* wf = full + warp * kTemniStages;
+  const int64_t gw = (int64_t)blockIdx.x * nwarps + warp, nw = (int64_t)gridDim.x * nwarps;
+  const int64_t n_my = (step > 0 && gw < rows) ? (rows - 1 - gw) / nw + 1 : 0;
+  const uint32_t row_bytes = (uint32_t)d * sizeof(float);
+  auto issue = [&](int64_t k) {
+    const int st = (int)(k % kTemniStages);
+    const int64_t row = gw + k * nw;
+    mbar_expect_tx(&wf[st], 2 * row_bytes);
+    bulk_load(wr + (size_t)st * 2 * d, xc + row * d, row_bytes, &wf[st]);
+    bulk_load(wr + (size_t)st * 2 * d + d, xp + row * d, row_bytes, &wf[st]);
+  };
+  if (lane == 0) {
+    for (int i = 0; i < kTemniStages; ++i) mbar_init(&wf[i], 1);
+    mbar_fence_init();
+    for (int64_t k = 0; k < n_my && k < kTemniStages; ++k) issue(k);
+  }
+  __syncthreads();  // modulation vectors staged, barriers initialised
+  const float inv_d = 1.0f / d;
   float num = 0.f, den = 0.f;
-  for (int64_t row = gw; row < rows; row += nw) {
-    const float* xr = x + row * d;
-    const float* pr = prev + row * d;
-    float v[NV][8];
-    float pe[kPrevEarly ? NV : 1][8];
+  int64_t k = 0;
+  for (; k < n_my; ++k) {
+    const int st = (int)(k % kTemniStages);
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(&wf[st], (uint32_t)((k / kTemniStages) & 1)));
+    if (!ok) break;
+    const float4* rc = reinterpret_cast<const float4*>(wr + (size_t)st * 2 * d);
+    const float4* rp = rc + d / 4;
+    // lane's vectors: i * 32 + lane, i < NV4 (4 columns each)
+    float4 cv[HOLD ? NV4 : 1], pv[HOLD ? NV4 : 1];
+    const float kc = wr[(size_t)st * 2 * d], kp = wr[(size_t)st * 2 * d + d];  // shifts: the rows' first elements
+    float s1c = 0.f, s2c = 0.f, s1p = 0.f, s2p = 0.f;
 #pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      const int c = (i * 32 + lane) * 8;
-      if (c < d) {
-        load8(xr + c, v[i]);
-        if constexpr (kPrevEarly) {
-          if (has_prev) load8(pr + c, pe[i]);
+    for (int i = 0; i < NV4; ++i) {
+      const int v = i * 32 + lane;
+      if (v < d / 4) {
+        const float4 c = rc[v], p = rp[v];
+        if constexpr (HOLD) {
+          cv[i] = c;
+          pv[i] = p;
+        }
+        const float c0 = c.x - kc, c1 = c.y - kc, c2 = c.z - kc, c3 = c.w - kc;
+        const float p0 = p.x - kp, p1 = p.y - kp, p2 = p.z - kp, p3 = p.w - kp;
+        s1c += (c0 + c1) + (c2 + c3);
+        s2c = fmaf(c0, c0, fmaf(c1, c1, fmaf(c2, c2, fmaf(c3, c3, s2c))));
+        s1p += (p0 + p1) + (p2 + p3);
+        s2p = fmaf(p0, p0, fmaf(p1, p1, fmaf(p2, p2, fmaf(p3, p3, s2p))));
+      }
+    }
+    if (HOLD) {
+      __syncwarp();
+      if (lane == 0 && k + kTemniStages < n_my) issue(k + kTemniStages);  // every lane holds its values
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      s1c += __shfl_xor_sync(0xffffffffu, s1c, o);
+      s2c += __shfl_xor_sync(0xffffffffu, s2c, o);
+      s1p += __shfl_xor_sync(0xffffffffu, s1p, o);
+      s2p += __shfl_xor_sync(0xffffffffu, s2p, o);
+    }
+    const float dc = s1c * inv_d, dp = s1p * inv_d;  // mean - K
+    const float mc = kc + dc, mp = kp + dp;
+    const float rsc = rsqrtf(fmaxf(s2c * inv_d - dc * dc, 0.f) + eps);
+    const float rsp = rsqrtf(fmaxf(s2p * inv_d - dp * dp, 0.f) + eps);
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+      const int v = i * 32 + lane;
+      if (v < d / 4) {
+        float4 c, p;
+        if constexpr (HOLD) {
+          c = cv[i];
+          p = pv[i];
+        } else {
+          c = rc[v];
+          p = rp[v];
+        }
+        const int q = d / 4;
+        const float4 bcv = mod[v], acv = mod[q + v], bpv = mod[2 * q + v], apv = mod[3 * q + v];
+        const float cc[4] = {c.x, c.y, c.z, c.w}, pp[4] = {p.x, p.y, p.z, p.w};
+        const float ac[4] = {acv.x, acv.y, acv.z, acv.w}, bc[4] = {bcv.x, bcv.y, bcv.z, bcv.w};
+        const float ap[4] = {apv.x, apv.y, apv.z, apv.w}, bp[4] = {bpv.x, bpv.y, bpv.z, bpv.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float uc = fmaf((cc[j] - mc) * rsc, ac[j], bc[j]);
+          const float up = fmaf((pp[j] - mp) * rsp, ap[j], bp[j]);
+          num += fabsf(uc - up);
+          den += fabsf(up);
         }
       }
     }
-    float s = 0.f;
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      const int c = (i * 32 + lane) * 8;
-      if (c < d) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) s += v[i][j];
-      }
-    }
-    const float mean = warp_sum_f(s) / d;
-    float q = 0.f;
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      const int c = (i * 32 + lane) * 8;
-      if (c < d) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float t = v[i][j] - mean;
-          q += t * t;
-        }
-      }
-    }
-    const float rstd = rsqrtf(warp_sum_f(q) / d + eps);
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      const int c = (i * 32 + lane) * 8;
-      if (c < d) {
-        float a[8], b[8];
-        load8(scale + c, a);
-        load8(shift + c, b);
-        float* o = v[i];  // the output replaces the input in place
-#pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = fmaf((o[j] - mean) * rstd, 1.0f + a[j], b[j]);
-        store8(cur + row * d + c, o);
-        if (has_prev) {
-          float pl[kPrevEarly ? 1 : 8];
-          const float* p = pl;
-          if constexpr (kPrevEarly) {
-            p = pe[i];
-          } else {
-            load8(pr + c, pl);
-          }
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            num += fabsf(o[j] - p[j]);
-            den += fabsf(p[j]);
-          }
-        }
-      }
+    if (!HOLD) {
+      __syncwarp();
+      if (lane == 0 && k + kTemniStages < n_my) issue(k + kTemniStages);  // every lane is done with the stage
     }
   }
-  __shared__ double sn[kThreads / 32], sd[kThreads / 32];
+  // after a wait ran out: the copies already issued land before the CTA exits
+  if (k < n_my && lane == 0)
+    for (int64_t j = k; j < n_my && j < k + kTemniStages; ++j)
+      mbar_wait(&wf[j % kTemniStages], (uint32_t)((j / kTemniStages) & 1));
   double dn = warp_sum_d((double)num), dd = warp_sum_d((double)den);
-  if (lane == 0) { sn[warp] = dn; sd[warp] = dd; }
+  if (lane == 0) {
+    rd[0][warp] = dn;
+    rd[1][warp] = dd;
+  }
   __syncthreads();
-  if (warp == 0) {
-    dn = lane < kThreads / 32 ? sn[lane] : 0.0;
-    dd = lane < kThreads / 32 ? sd[lane] : 0.0;
-    dn = warp_sum_d(dn);
-    dd = warp_sum_d(dd);
-    if (lane == 0) partials[blockIdx.x] = make_double2(dn, dd);
+  if (threadIdx.x == 0) {
+    dn = 0.0;
+    dd = 0.0;
+    for (int w = 0; w < nwarps; ++w) {
+      dn += rd[0][w];
+      dd += rd[1][w];
+    }
+    partials[blockIdx.x] = make_double2(dn, dd);
   }
 }
 
@@ -632,25 +708,51 @@ acid_status ln_mod(int in_dtype, const void* x, int out_dtype, void* y, int64_t 
   return launch_ln_mod<kLnMaxV>(in_dtype, out_dtype, x, y, rows, d, shv, scv, sht, sct, split, eps, blocks, s);
 }
 
-acid_status ln_mod_drift(const float* x, float* tem0, float* tem1, const int* step_dev, int step_host, int64_t rows,
-                         int d, const float* shift, const float* scale, float eps, double* d_result, void* workspace,
-                         size_t ws_bytes, cudaStream_t s) {
-  ACID_REQUIRE(d % 8 == 0 && d <= 256 * kLnMaxV, ACID_ERR_UNSUPPORTED, "ln_mod_drift: d must be a multiple of 8, <= 3072");
-  ACID_REQUIRE(ws_bytes >= sizeof(double2) * kDriftMaxBlocks, ACID_ERR_WORKSPACE, "ln_mod_drift: workspace too small");
-  double2* parts = static_cast<double2*>(workspace);
-  const int64_t want = (rows * 32 + kThreads - 1) / kThreads;
-  const int grid = (int)std::min<int64_t>(kDriftMaxBlocks, std::max<int64_t>(1, want));
-  ProfScope prof(PROF_DRIFT, (double)rows * d * 12.0, s);  // read x and prev, write cur (fp32)
-  if (d <= 256 * 4)
-    ln_mod_drift_kernel<4><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
-  else if (d <= 256 * 6)
-    ln_mod_drift_kernel<6><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
-  else if (d <= 256 * 8)
-    ln_mod_drift_kernel<8><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale, eps, parts);
-  else
-    ln_mod_drift_kernel<kLnMaxV><<<grid, kThreads, 0, s>>>(x, tem0, tem1, step_dev, step_host, rows, d, shift, scale,
-                                                           eps, parts);
+template <int NV4, bool HOLD>
+acid_status launch_temni_drift(const float* h_cur, const float* h_prev, const float* mod_cur, const float* mod_prev,
+                               const int* step_dev, int step_host, int64_t rows, int d, float eps, double2* parts,
+                               cudaStream_t s, int* grid_out) {
+  constexpr int kSmemMax = 226 * 1024;  // dynamic shared memory, below the 227 KB limit less the static part
+  static bool attr_done = false;
+  if (!attr_done) {
+    ACID_CUDA(cudaFuncSetAttribute(temni_drift_kernel<NV4, HOLD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemMax));
+    attr_done = true;
+  }
+  // warps per CTA: as many two-stage rings (8 d bytes per stage) as fit
+  // beside the staged modulation vectors (16 d bytes), at most eight
+  const size_t ring_per_warp = (size_t)kTemniStages * 8 * d + kTemniStages * sizeof(uint64_t);
+  const int warps = (int)std::max<size_t>(1, std::min<size_t>(kTemniMaxWarps, (kSmemMax - 16 * (size_t)d) /
+                                                                                   ring_per_warp));
+  const size_t smem = 16 * (size_t)d + warps * ring_per_warp;
+  const int grid = (int)std::min<int64_t>(std::min<int64_t>(kDriftMaxBlocks, (int64_t)num_sms_elem()),
+                                          std::max<int64_t>(1, (rows + warps - 1) / warps));
+  temni_drift_kernel<NV4, HOLD><<<grid, 32 * warps, smem, s>>>(h_cur, h_prev, step_dev, step_host, rows, d, mod_cur,
+                                                               mod_cur + d, mod_prev, mod_prev + d, eps, parts);
   ACID_CHECK_LAUNCH();
+  *grid_out = grid;
+  return ACID_OK;
+}
+
+acid_status temni_drift(const float* h_cur, const float* h_prev, const float* mod_cur, const float* mod_prev,
+                        const int* step_dev, int step_host, int64_t rows, int d, float eps, double* d_result,
+                        void* workspace, size_t ws_bytes, cudaStream_t s) {
+  ACID_REQUIRE(d % 8 == 0 && d <= 3072, ACID_ERR_UNSUPPORTED, "temni_drift: d must be a multiple of 8, <= 3072");
+  ACID_REQUIRE(ws_bytes >= sizeof(double2) * kDriftMaxBlocks, ACID_ERR_WORKSPACE, "temni_drift: workspace too small");
+  ACID_REQUIRE(aligned(h_cur, 16) && aligned(h_prev, 16) && aligned(mod_cur, 16) && aligned(mod_prev, 16),
+               ACID_ERR_UNSUPPORTED, "temni_drift: inputs must be 16-byte aligned");
+  double2* parts = static_cast<double2*>(workspace);
+  ProfScope prof(PROF_DRIFT, (double)rows * d * 8.0, s);  // read both steps' H_in (fp32)
+  int grid = 1;
+  if (d <= 512)
+    ACID_TRY((launch_temni_drift<4, true>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts, s,
+                                         &grid)));
+  else if (d <= 1536)
+    ACID_TRY((launch_temni_drift<12, true>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts,
+                                          s, &grid)));
+  else
+    ACID_TRY((launch_temni_drift<24, false>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts,
+                                           s, &grid)));
   drift_final_kernel<<<1, kThreads, 0, s>>>(parts, grid, d_result);
   ACID_CHECK_LAUNCH();
   return ACID_OK;

@@ -149,7 +149,7 @@ struct TcCfg {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int EPI_STAGE_FLOATS = 32 * 33;  // one 32x32 chunk per epilogue warp, padded rows
+  static constexpr int EPI_STAGE_FLOATS = 32 * 32;  // one 32x32 chunk per epilogue warp (swizzled units)
   static constexpr int EPI_BYTES = kEpiWarps * EPI_STAGE_FLOATS * 4;
   static constexpr int SMEM = STAGES * STAGE_BYTES + EPI_BYTES + 1024 + 256;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
@@ -195,7 +195,11 @@ __device__ __forceinline__ void load_chunk_inputs(const GemmDims& g, const EpiDe
 #pragma unroll
     for (int p = 0; p < 8; ++p) {
       const int64_t row = row0 + 4 * p + (lane >> 3);
-      if (row >= g.M) continue;
+      if (row >= g.M) {  // computed but not stored by the epilogue
+#pragma unroll
+        for (int q = 0; q < (R32 ? 4 : 2); ++q) rc.w[p][q] = 0u;
+        continue;
+      }
       if constexpr (R32) {
         const uint4 t = *reinterpret_cast<const uint4*>(static_cast<const float*>(e.res) + row * e.ldr + col);
         rc.w[p][0] = t.x; rc.w[p][1] = t.y; rc.w[p][2] = t.z; rc.w[p][3] = t.w;
@@ -217,12 +221,36 @@ __device__ __forceinline__ float res_value(const ResChunk<R32>& rc, int p, int k
   }
 }
 
+// GELU (tanh form) of a packed pair, with the arithmetic of gelu_tanh<true>
+// done two lanes at a time: u = sqrt(2/pi) (x + 0.044715 x^3), out = h + h tanh(u)
+// with h = x / 2.
+__device__ __forceinline__ uint64_t gelu_x2(uint64_t x) {
+  const uint64_t c3 = f2_pack(0.044715f, 0.044715f), k0 = f2_pack(0.7978845608028654f, 0.7978845608028654f);
+  const uint64_t half = f2_pack(0.5f, 0.5f);
+  const uint64_t u = f2_mul(k0, f2_fma(f2_mul(c3, x), f2_mul(x, x), x));
+  float u0, u1;
+  f2_unpack(u, u0, u1);
+  const uint64_t t = f2_pack(tanh_fast(u0), tanh_fast(u1));
+  const uint64_t h = f2_mul(half, x);
+  return f2_fma(h, t, h);
+}
+
+// The stage of one epilogue warp: 32 rows x 32 fp32 columns, row-major, the
+// eight 16-byte units of row r stored in the order u ^ (r & 7), so that both
+// the row-wise writes (lane = row) and the transposed reads (8 lanes per row)
+// touch every bank once per 128 bytes.
+__device__ __forceinline__ float4* stage_unit(float* stage, int row, int unit) {
+  return reinterpret_cast<float4*>(stage) + row * 8 + (unit ^ (row & 7));
+}
+
 template <int KIND, bool R32>
 __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, float* stage, int64_t row0,
                                                int col0, const uint32_t* r, const ResChunk<R32>& rc) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int j = 0; j < 32; ++j) stage[lane * 33 + j] = __uint_as_float(r[j]);
+  for (int u = 0; u < 8; ++u)
+    *stage_unit(stage, lane, u) = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
+                                              __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
   __syncwarp();
   const int c = 4 * (lane & 7);
   const int col = col0 + c;
@@ -243,23 +271,28 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
       }
     }
   }
+  const uint64_t b01 = f2_pack(rc.bias[0], rc.bias[1]), b23 = f2_pack(rc.bias[2], rc.bias[3]);
+  // rows past M are computed like the others (from whatever the stage and
+  // residual registers hold) and only their stores are skipped, so the eight
+  // row groups form one branch-free block the compiler can interleave
 #pragma unroll
   for (int p = 0; p < 8; ++p) {
     const int rr = 4 * p + (lane >> 3);
     const int64_t row = row0 + rr;
-    if (row >= g.M) continue;
     const int64_t grow = row + e.row_base;
-    float v[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) v[k] = stage[rr * 33 + c + k] + rc.bias[k];
+    const float4 sv = *stage_unit(stage, rr, lane & 7);
+    uint64_t v01 = f2_add(f2_pack(sv.x, sv.y), b01), v23 = f2_add(f2_pack(sv.z, sv.w), b23);
     switch (KIND) {
       case EPI_GELU:
-#pragma unroll
-        for (int k = 0; k < 4; ++k) v[k] = gelu_tanh<true>(v[k]);
+        v01 = gelu_x2(v01);
+        v23 = gelu_x2(v23);
         break;
-      case EPI_ROPE_QKV:
+      case EPI_ROPE_QKV: {
         // (cos, sin) = (1, 0) on rows and columns that are not rotated; the
         // four columns lie in one head (head_dim is a power of two)
+        float v[4];
+        f2_unpack(v01, v[0], v[1]);
+        f2_unpack(v23, v[2], v[3]);
 #pragma unroll
         for (int k = 0; k < 4; k += 2) {
           const float2 cs = rcs[p][k >> 1];
@@ -267,20 +300,29 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
           v[k] = x0 * cs.x - x1 * cs.y;
           v[k + 1] = x0 * cs.y + x1 * cs.x;
         }
+        v01 = f2_pack(v[0], v[1]);
+        v23 = f2_pack(v[2], v[3]);
         break;
+      }
       case EPI_GATED_RES: {
         const bool text = grow < e.gate_split;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) v[k] = fmaf(text ? rc.gt[k] : rc.gv[k], v[k], res_value(rc, p, k));
+        const uint64_t g01 = text ? f2_pack(rc.gt[0], rc.gt[1]) : f2_pack(rc.gv[0], rc.gv[1]);
+        const uint64_t g23 = text ? f2_pack(rc.gt[2], rc.gt[3]) : f2_pack(rc.gv[2], rc.gv[3]);
+        v01 = f2_fma(g01, v01, f2_pack(res_value(rc, p, 0), res_value(rc, p, 1)));
+        v23 = f2_fma(g23, v23, f2_pack(res_value(rc, p, 2), res_value(rc, p, 3)));
         break;
       }
       case EPI_RES:
-#pragma unroll
-        for (int k = 0; k < 4; ++k) v[k] += res_value(rc, p, k);
+        v01 = f2_add(v01, f2_pack(res_value(rc, p, 0), res_value(rc, p, 1)));
+        v23 = f2_add(v23, f2_pack(res_value(rc, p, 2), res_value(rc, p, 3)));
         break;
       default:
         break;
     }
+    float v[4];
+    f2_unpack(v01, v[0], v[1]);
+    f2_unpack(v23, v[2], v[3]);
+    if (row >= g.M) continue;
     if (g.out_fp32)
       *reinterpret_cast<float4*>(static_cast<float*>(g.out) + row * g.ldo + col) = make_float4(v[0], v[1], v[2], v[3]);
     else
@@ -430,6 +472,195 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   }
 }
 
+// ===========================================================================
+// tcgen05 GEMM on SM pairs (cta_group::2), persistent
+//
+// A cluster of two CTAs on two SMs computes 256 x 256 output tiles: each CTA
+// stages its own 128 rows of A and its own 128 rows of B (half of the tile's
+// output columns) per 64-wide k-step, and one thread of CTA rank 0 issues
+// M256 N256 K16 MMAs that read both CTAs' shared memory and write each CTA's
+// 128 x 256 fp32 accumulator into that CTA's TMEM.  Per SM and k-step this
+// moves 32 KB into shared memory for 128 x 256 x 64 MACs, against 48 KB for
+// the single-SM 128 x 256 tile: the single-SM kernel is bound by that
+// L2-to-SM delivery.
+//   warp 0   TMA producer in both CTAs; both CTAs' loads count on rank 0's
+//            full[s] barrier (rank 0 expects the bytes of both);
+//   warp 1   rank 0: MMA issuer; each k-step is committed to empty[s] of both
+//            CTAs, each tile to acc_full[b] of both CTAs;
+//   warps 2-9 epilogue of this CTA's 128 accumulator rows (as in
+//            gemm_tc_kernel); one lane per warp then arrives on rank 0's
+//            acc_empty[b], which counts the epilogue warps of both CTAs.
+// ===========================================================================
+struct Tc2Cfg {
+  static constexpr int BN = 256;  // output columns per pair tile
+  static constexpr int STAGES = 6;
+  static constexpr int A_BYTES = BM * BK * 2;        // this CTA's 128 rows of A
+  static constexpr int B_BYTES = (BN / 2) * BK * 2;  // this CTA's 128 rows of B
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int EPI_STAGE_FLOATS = 32 * 32;
+  static constexpr int EPI_BYTES = kEpiWarps * EPI_STAGE_FLOATS * 4;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + EPI_BYTES + 1024 + 256;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // double-buffered 128 x 256 accumulator
+};
+static_assert(Tc2Cfg::SMEM <= 232448, "pair GEMM shared memory");
+
+template <int KIND, bool R32>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
+                    EpiDev e) {
+  using C = Tc2Cfg;
+  constexpr int BN = C::BN;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES + C::EPI_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* acc_full = empty + C::STAGES;  // [2]
+  uint64_t* acc_empty = acc_full + 2;      // [2] (rank 0's counts both CTAs' epilogue warps)
+  uint64_t* drain = acc_empty + 2;         // failure path: the MMAs issued so far have completed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = (int)blockIdx.x >> 1, npairs = (int)gridDim.x >> 1;
+  const int num_kb = (g.K + BK - 1) / BK;
+  const int num_n = (g.N + BN - 1) / BN;
+  const int num_tiles = (int)((g.M + 2 * BM - 1) / (2 * BM)) * num_n;
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 2 * kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_slot, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs' barriers exist before any cross-CTA arrival
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // TMA producer (both CTAs): one continuous stage ring across tiles
+      const uint32_t full0 = mapa_shared(smem_u32(full), 0);  // rank 0's full[0]
+      int it = 0;
+      bool ok = true;
+      for (int tile = pair; ok && tile < num_tiles; tile += npairs) {
+        const int m_tile = tile / num_n, n_tile = tile % num_n;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % C::STAGES, round = it / C::STAGES;
+          if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1)) { ok = false; break; }
+          if (rank == 0) mbar_expect_tx(&full[s], 2 * C::STAGE_BYTES);
+          tma_load_2d_pair(sA + s * C::A_BYTES, &tmA, full0 + 8 * s, kb * BK, m_tile * 2 * BM + (int)rank * BM);
+          tma_load_2d_pair(sB + s * C::B_BYTES, &tmB, full0 + 8 * s, kb * BK, n_tile * BN + (int)rank * (BN / 2));
+        }
+      }
+      // After a wait ran out: rank 0 waits (bounded) for the last STAGES
+      // stages it expected to land.  Rank 1's loads count on rank 0's
+      // barriers, which rank 1 cannot poll; it idles about 2^16 clocks, far
+      // above the latency of a 32 KB load, before both CTAs meet at the exit.
+      if (!ok) {
+        if (rank == 0) {
+          for (int j = std::max(0, it - C::STAGES); j < it; ++j) mbar_wait(&full[j % C::STAGES], (j / C::STAGES) & 1);
+        } else {
+          const long long t0 = clock64();
+          while (clock64() - t0 < (1LL << 16)) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {  // MMA issuer (rank 0 only)
+      constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, BN, false, false);
+      const uint32_t empty_l = smem_u32(empty), empty_r = mapa_shared(empty_l, 1);
+      const uint32_t accf_l = smem_u32(acc_full), accf_r = mapa_shared(accf_l, 1);
+      int it = 0, local = 0;
+      bool ok = true;
+      for (int tile = pair; ok && tile < num_tiles; tile += npairs, ++local) {
+        const int b = local & 1, use = local >> 1;
+        if (use > 0 && !mbar_wait_cluster(&acc_empty[b], (use - 1) & 1)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d = tmem + b * BN;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % C::STAGES, round = it / C::STAGES;
+          if (!mbar_wait(&full[s], round & 1)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t ad = smem_desc_sw128(a0 + k * 32, 16, 1024);
+            const uint64_t bd = smem_desc_sw128(b0 + k * 32, 16, 1024);
+            mma_bf16_ss_pair(d, ad, bd, idesc, (kb | k) != 0);
+          }
+          mma_commit_pair(empty_l + 8 * s);
+          mma_commit_pair(empty_r + 8 * s);
+        }
+        if (ok) {
+          mma_commit_pair(accf_l + 8 * b);
+          mma_commit_pair(accf_r + 8 * b);
+        }
+      }
+      if (!ok) {
+        mma_commit_pair(smem_u32(drain));
+        mbar_wait(drain, 0);
+      }
+    }
+  } else {  // epilogue: warps 2..9 of each CTA, this CTA's 128 rows of the pair tile
+    const int q = warp & 3, half = (warp - 2) >> 2;
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    float* stage = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES) + (warp - 2) * C::EPI_STAGE_FLOATS;
+    const uint32_t acc_empty0 = mapa_shared(smem_u32(acc_empty), 0);
+    int local = 0;
+    for (int tile = pair; tile < num_tiles; tile += npairs, ++local) {
+      const int b = local & 1, use = local >> 1;
+      const int m_tile = tile / num_n, n_tile = tile % num_n;
+      const bool ok = mbar_wait(&acc_full[b], use & 1);
+      tc_fence_after();
+      const int64_t row0 = (int64_t)m_tile * 2 * BM + (int64_t)rank * BM + q * 32;
+      constexpr int NC = BN / 64;
+      const int cbeg = half * (BN / 2);
+      const int lcol = 4 * (lane & 7);
+      auto process = [&](int i, const ResChunk<R32>& cur, ResChunk<R32>& nxt) {
+        const int c = cbeg + 32 * i;
+        uint32_t r[32];
+        tmem_ld32(tmem + lane_base + b * BN + c, r);
+        tmem_wait_ld();
+        const int col0 = n_tile * BN + c;
+        if (i + 1 < NC && row0 < g.M && col0 + 32 < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, col0 + 32 + lcol, nxt);
+        if (ok && row0 < g.M && col0 < g.N) epilogue_chunk<KIND, R32>(g, e, stage, row0, col0, r, cur);
+      };
+      ResChunk<R32> rc0, rc1;
+      if (row0 < g.M && n_tile * BN + cbeg < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, n_tile * BN + cbeg + lcol, rc0);
+#pragma unroll 1
+      for (int i = 0; i < NC; i += 2) {
+        process(i, rc0, rc1);
+        if (i + 1 < NC) process(i + 1, rc1, rc0);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc_empty0 + 8 * b);
+      if (!ok) break;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal its barriers
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, C::TMEM_COLS);
+  }
+}
+
 // ---------------------------------------------------------------------------
 // TMA descriptor encoding through the driver entry point (no -lcuda needed)
 // ---------------------------------------------------------------------------
@@ -519,6 +750,60 @@ acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* 
       return epi.res_fp32 ? launch_tc_kind<BN, EPI_RES, true>(ta, tb, g, epi, grid, s)
                           : launch_tc_kind<BN, EPI_RES, false>(ta, tb, g, epi, grid, s);
     default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, g, epi, grid, s);
+  }
+}
+
+// CTA pairs that can be resident at once for the pair kernel (clusters are
+// placed within a GPC, so this can be below half the SM count).
+template <int KIND, bool R32>
+int max_pairs() {
+  static int n = -1;
+  if (n < 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * 76, 1, 1);
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = Tc2Cfg::SMEM;
+    int c = 0;
+    n = (cudaOccupancyMaxActiveClusters(&c, gemm_tc2_kernel<KIND, R32>, &cfg) == cudaSuccess && c > 0) ? c : 0;
+  }
+  return n;
+}
+
+template <int KIND, bool R32 = false>
+acid_status launch_tc2_kind(const CUtensorMap& ta, const CUtensorMap& tb, const GemmDims& g, const Epilogue& epi,
+                            int64_t tiles, cudaStream_t s) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    ACID_CUDA(cudaFuncSetAttribute(gemm_tc2_kernel<KIND, R32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   Tc2Cfg::SMEM));
+    attr_done = true;
+  }
+  const int pairs = max_pairs<KIND, R32>();
+  ACID_REQUIRE(pairs > 0, ACID_ERR_CUDA, "linear: no resident CTA pair for the pair GEMM");
+  const int grid = 2 * (int)std::min<int64_t>(tiles, pairs);
+  gemm_tc2_kernel<KIND, R32><<<grid, kGemmThreads, Tc2Cfg::SMEM, s>>>(ta, tb, g, to_dev(epi));
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status launch_tc2(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
+                       const Epilogue& epi, cudaStream_t s) {
+  CUtensorMap ta, tb;
+  ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
+  ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, Tc2Cfg::BN / 2));
+  GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0};
+  const int64_t tiles = ((M + 2 * BM - 1) / (2 * BM)) * ((N + Tc2Cfg::BN - 1) / Tc2Cfg::BN);
+  ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
+  switch (epi.kind) {
+    case EPI_GELU: return launch_tc2_kind<EPI_GELU>(ta, tb, g, epi, tiles, s);
+    case EPI_ROPE_QKV: return launch_tc2_kind<EPI_ROPE_QKV>(ta, tb, g, epi, tiles, s);
+    case EPI_GATED_RES:
+      return epi.res_fp32 ? launch_tc2_kind<EPI_GATED_RES, true>(ta, tb, g, epi, tiles, s)
+                          : launch_tc2_kind<EPI_GATED_RES, false>(ta, tb, g, epi, tiles, s);
+    case EPI_RES:
+      return epi.res_fp32 ? launch_tc2_kind<EPI_RES, true>(ta, tb, g, epi, tiles, s)
+                          : launch_tc2_kind<EPI_RES, false>(ta, tb, g, epi, tiles, s);
+    default: return launch_tc2_kind<EPI_BIAS>(ta, tb, g, epi, tiles, s);
   }
 }
 
@@ -627,6 +912,11 @@ acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int
   // shared-memory bytes per FLOP than a 256-wide one, which costs more than
   // the zero-filled columns of a partial last tile (N = 1920: 7% extra MMA
   // work, against about 1.6x the throughput).
+  // SM pairs where the tiles' mainloop is long enough to matter: measured at
+  // M = 32760, pairs are 1-2% faster for N = 4608 / 8960 or K = 8960 and 3%
+  // slower for the 1536 x 1536 output projection, whose fp32 residual traffic
+  // bounds it as much as its FLOPs do.
+  if (N > 128 && (N > 2048 || K > 2048)) return launch_tc2(A, lda, M, K, W, N, out, ldo, epi, s);
   if (N > 128) return launch_tc<256>(A, lda, M, K, W, N, out, ldo, epi, s);
   if (N > 64) return launch_tc<128>(A, lda, M, K, W, N, out, ldo, epi, s);
   return launch_tc<64>(A, lda, M, K, W, N, out, ldo, epi, s);

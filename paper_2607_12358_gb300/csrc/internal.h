@@ -84,6 +84,15 @@ acid_status ln_mod(int in_dtype, const void* x, int out_dtype, void* y, int64_t 
                    const float* shift_v, const float* scale_v, const float* shift_t,
                    const float* scale_t, int64_t split, float eps, cudaStream_t s);
 
+// TeaCache signal sums from the fp32 patch embeddings of two consecutive steps
+// and their block-0 modulations (shift then scale, d each): TEMNI of both
+// steps formed in registers, 8 bytes read per element.  Result {rel, num, den}
+// in d_result as drift_launch.  step from step_dev (device) if non-null, else
+// step_host; step 0 gives zero sums.
+acid_status temni_drift(const float* h_cur, const float* h_prev, const float* mod_cur, const float* mod_prev,
+                        const int* step_dev, int step_host, int64_t rows, int d, float eps, double* d_result,
+                        void* workspace, size_t ws_bytes, cudaStream_t s);
+
 // y[j] = sum_k W[j, k] act(x[k]) + b[j]; act = SiLU if silu_input.
 acid_status gemv(int w_dtype, const void* W, const float* b, const float* x, float* y, int n_out,
                  int k, bool silu_input, cudaStream_t s);
@@ -95,13 +104,6 @@ size_t drift_workspace_bytes(int64_t n);
 acid_status drift_launch(int dtype, const void* prev, const void* cur, const void* resid, void* out,
                          int64_t n, double* d_result /* device double[3]: rel, num, den */,
                          void* workspace, size_t ws_bytes, cudaStream_t s);
-
-// TEMNI = LN(x) (1 + scale) + shift written to tem[step & 1] (fp32), and the
-// relative-L1 drift against tem[(step + 1) & 1] in the same pass; result as
-// drift_launch.  step from step_dev (device) if non-null, else step_host.
-acid_status ln_mod_drift(const float* x, float* tem0, float* tem1, const int* step_dev, int step_host, int64_t rows,
-                         int d, const float* shift, const float* scale, float eps, double* d_result, void* workspace,
-                         size_t ws_bytes, cudaStream_t s);
 
 // out = a + b elementwise, one dtype, 16-byte vectors
 acid_status add_same(int dtype, const void* a, const void* b, void* out, int64_t n, cudaStream_t s);

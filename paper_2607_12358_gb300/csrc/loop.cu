@@ -26,11 +26,11 @@ struct LoopWs {
   float* sinus;
   float* temb_h;
   float* temb;
-  float* mod0;      // block 0 shift / scale (TEMNI)
+  float* mod0[2];   // block 0 shift / scale (TEMNI) of the even / odd steps
   float* fmod;      // final layer shift / scale
   uint8_t* tokens;  // [N, P] fp32 patch vectors
-  float* h_in;      // [N, d] patch embedding (fp32)
-  float* temni[2];  // [N, d] block-0 modulated input, current / previous
+  float* h_in[2];   // [N, d] patch embedding (fp32) of the even / odd steps
+  float* temni[2];  // [N, d] DiCache probe features of the even / odd steps
   float* resid;     // [N, d] TeaCache residual H_out - H_in
   uint8_t* xbuf;    // [L + N, d] block-stack state (model dtype)
   uint8_t* text;    // [L, d] text context / text tokens (model dtype)
@@ -110,10 +110,12 @@ LoopWs loop_layout(const acid_model& m, void* base) {
   w.sinus = b.take<float>(m.time_freq_dim);
   w.temb_h = b.take<float>(s.d);
   w.temb = b.take<float>(s.d);
-  w.mod0 = b.take<float>(2 * s.d);
+  w.mod0[0] = b.take<float>(2 * s.d);
+  w.mod0[1] = b.take<float>(2 * s.d);
   w.fmod = b.take<float>(2 * s.d);
   w.tokens = b.take<uint8_t>(s.N * s.P * sizeof(float));
-  w.h_in = b.take<float>(s.N * s.d);
+  w.h_in[0] = b.take<float>(s.N * s.d);
+  w.h_in[1] = b.take<float>(s.N * s.d);
   w.temni[0] = b.take<float>(s.N * s.d);
   w.temni[1] = b.take<float>(s.N * s.d);
   w.resid = b.take<float>(s.N * s.d);
@@ -475,6 +477,9 @@ static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, ac
   const double t = 1000.0 * sig;
   const float dsig = (float)(sig_next - sig);
   const bool warm = i < cfg->warmup;
+  // buffers of this step and of the previous one alternate with the parity
+  const int par = i & 1;
+  float* h_in = w.h_in[par];
   int forced = cfg->forced ? cfg->forced[i] : -1;
   if (forced < 0 && cfg->force_last && i == cfg->n_steps - 1) forced = 1;
   memset(&lg, 0, sizeof(lg));
@@ -496,24 +501,24 @@ static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, ac
     Epilogue e;
     e.bias = m->patch.b;
     e.out_fp32 = true;
-    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m->patch.w, sh.d, w.h_in, sh.d, e, s));
+    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m->patch.w, sh.d, h_in, sh.d, e, s));
   }
   const int64_t vrow0 = m->block.kind == ACID_BLOCK_WAN ? 0 : sh.L;
   void* x_video = w.xbuf + vrow0 * sh.d * es(dt);
   auto run_model = [&]() -> acid_status {
     if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
-    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
+    ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
     return run_blocks(*m, w, s);
   };
 
   bool compute = true;
   if (cfg->method == ACID_METHOD_TEACACHE) {
-    // s_t: rel_l1 of block 0's modulated input between consecutive steps
-    // TEMNI_i = block 0's modulated input, written to temni[i & 1], and its
-    // drift against TEMNI_{i-1} in temni[(i + 1) & 1], in one pass
-    ACID_TRY(gemv(dt, m->blocks[0].mod.w, m->blocks[0].mod.b, w.temb, w.mod0, 2 * sh.d, sh.d, true, s));
-    ACID_TRY(ln_mod_drift(w.h_in, w.temni[0], w.temni[1], nullptr, i, sh.N, sh.d, w.mod0, w.mod0 + sh.d,
-                          m->block.ln_eps, w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+    // s_t: rel_l1 of block 0's modulated input (TEMNI) between consecutive
+    // steps, both TEMNIs formed from this and the previous step's H_in and
+    // block-0 modulation in one read-only pass
+    ACID_TRY(gemv(dt, m->blocks[0].mod.w, m->blocks[0].mod.b, w.temb, w.mod0[par], 2 * sh.d, sh.d, true, s));
+    ACID_TRY(temni_drift(h_in, w.h_in[par ^ 1], w.mod0[par], w.mod0[par ^ 1], nullptr, i, sh.N, sh.d,
+                         m->block.ln_eps, w.dres, w.drift_ws, drift_workspace_bytes(0), s));
     if (!warm) {
       ACID_REQUIRE(i > 0, ACID_ERR_INVALID_ARG, "TeaCache needs at least one warmup step");
       double h[3];
@@ -523,20 +528,20 @@ static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, ac
     if (compute || !st->have_cache) {
       compute = true;
       ACID_TRY(run_model());
-      ACID_TRY(add_mixed(dt, x_video, ACID_FP32, w.h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s));
+      ACID_TRY(add_mixed(dt, x_video, ACID_FP32, h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s));
       st->have_cache = 1;
     } else {
-      ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s));
+      ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s));
     }
     ACID_TRY(final_layer(*m, w, x_video, defer_euler ? w.v[0] : nullptr, defer_euler ? nullptr : latent, dsig, s));
     if (defer_euler) *v_out = w.v[0];
   } else if (cfg->method == ACID_METHOD_DICACHE) {
     // probe: the first probe_blocks blocks on every step; P_i (fp32) in temni[i & 1]
     const int pb = cfg->probe_blocks;
-    float* p_cur = w.temni[i & 1];
-    float* p_prev = w.temni[(i & 1) ^ 1];
+    float* p_cur = w.temni[par];
+    float* p_prev = w.temni[par ^ 1];
     if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
-    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
+    ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
     ACID_TRY(run_blocks(*m, w, s, 0, pb));
     ACID_TRY(add_mixed(dt, x_video, dt, x_video, ACID_FP32, p_cur, sh.N * sh.d, 0.0f, s));
     if (!warm) {
@@ -828,18 +833,20 @@ struct GraphCapture {
 };
 
 // Records, into the graph `body` that gc.main is capturing, one branch's part
-// of a step: its inputs, signal and Algorithm 1 decision, the compute or reuse
-// body of an IF/ELSE node (captured on gc.side), and its velocity in w.v[0]
-// together with the copies that keep the previous step's values.  The Euler
-// update is left to the caller.
+// of a step of parity `par` (the buffers that alternate between steps are
+// chosen here; the graph holds one such body per parity): its inputs, signal
+// and Algorithm 1 decision, the compute or reuse body of an IF/ELSE node
+// (captured on gc.side), and its velocity in w.v[0] together with the copies
+// that keep the previous step's values.  The Euler update is left to the caller.
 acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& w, float* latent,
-                           GraphCapture& gc, cudaGraph_t body) {
+                           GraphCapture& gc, cudaGraph_t body, int par) {
   const Shape sh = shape_of(m);
   const int dt = m.block.dtype;
   cudaStream_t s = gc.main, s2 = gc.side;
   const int* step = &w.dev->step;
   const int64_t vrow0 = m.block.kind == ACID_BLOCK_WAN ? 0 : sh.L;
   void* x_video = w.xbuf + vrow0 * sh.d * es(dt);
+  float* h_in = w.h_in[par];
   cudaGraphConditionalHandle h_compute;
   ACID_CUDA(cudaGraphConditionalHandleCreate(&h_compute, body, 0, 0));
 
@@ -852,22 +859,22 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
     Epilogue e;
     e.bias = m.patch.b;
     e.out_fp32 = true;
-    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m.patch.w, sh.d, w.h_in, sh.d, e, s));
+    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m.patch.w, sh.d, h_in, sh.d, e, s));
   }
   // ---- signal and decision
   float* v = w.v[0];
   float* v_prev = w.v[1];
-  // DiCache probe features: current in temni[0], previous step's in temni[1]
-  float* p_cur = w.temni[0];
-  float* p_prev = w.temni[1];
+  // DiCache probe features of this step and of the previous one
+  float* p_cur = w.temni[par];
+  float* p_prev = w.temni[par ^ 1];
   const int pb = cfg.probe_blocks;
   if (cfg.method == ACID_METHOD_TEACACHE) {
-    ACID_TRY(gemv(dt, m.blocks[0].mod.w, m.blocks[0].mod.b, w.temb, w.mod0, 2 * sh.d, sh.d, true, s));
-    ACID_TRY(ln_mod_drift(w.h_in, w.temni[0], w.temni[1], step, 0, sh.N, sh.d, w.mod0, w.mod0 + sh.d, m.block.ln_eps,
-                          w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+    ACID_TRY(gemv(dt, m.blocks[0].mod.w, m.blocks[0].mod.b, w.temb, w.mod0[par], 2 * sh.d, sh.d, true, s));
+    ACID_TRY(temni_drift(h_in, w.h_in[par ^ 1], w.mod0[par], w.mod0[par ^ 1], step, 0, sh.N, sh.d, m.block.ln_eps,
+                         w.dres, w.drift_ws, drift_workspace_bytes(0), s));
   } else if (cfg.method == ACID_METHOD_DICACHE) {
     if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
-    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
+    ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, h_in, dt, x_video, sh.N * sh.d, 0.0f, s));
     ACID_TRY(run_blocks(m, w, s, 0, pb));
     ACID_TRY(add_mixed(dt, x_video, dt, x_video, ACID_FP32, p_cur, sh.N * sh.d, 0.0f, s));
     ACID_TRY(drift_launch(ACID_FP32, p_prev, p_cur, nullptr, nullptr, sh.N * sh.d, w.dres, w.drift_ws,
@@ -890,12 +897,12 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
     ACID_TRY(dicache_update(dt, x_video, p_cur, w, sh.N * sh.d, s2));
   } else {
     if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s2));
-    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.h_in, dt, x_video, sh.N * sh.d, 0.0f, s2));
+    ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, h_in, dt, x_video, sh.N * sh.d, 0.0f, s2));
     ACID_TRY(run_blocks(m, w, s2));
   }
   if (cfg.method == ACID_METHOD_DICACHE) {
   } else if (cfg.method == ACID_METHOD_TEACACHE) {
-    ACID_TRY(add_mixed(dt, x_video, ACID_FP32, w.h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s2));
+    ACID_TRY(add_mixed(dt, x_video, ACID_FP32, h_in, ACID_FP32, w.resid, sh.N * sh.d, -1.0f, s2));
   } else {
     ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s2));
     ACID_TRY(drift_launch(ACID_FP32, v_prev, v, nullptr, nullptr, sh.latent, w.dres, w.drift_ws,
@@ -911,7 +918,7 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
   // ---- reuse body: cached residual / offset
   ACID_CUDA(cudaStreamBeginCaptureToGraph(s2, br[1], nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
   if (cfg.method == ACID_METHOD_TEACACHE)
-    ACID_TRY(add_mixed(ACID_FP32, w.h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s2));
+    ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, w.resid, dt, x_video, sh.N * sh.d, 1.0f, s2));
   else if (cfg.method == ACID_METHOD_DICACHE)
     ACID_TRY(dicache_reuse(dt, x_video, p_cur, w, sh.N * sh.d, s2));
   else
@@ -923,7 +930,6 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
     ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s));
   } else if (cfg.method == ACID_METHOD_DICACHE) {
     ACID_TRY(final_layer(m, w, x_video, v, nullptr, 0.0f, s));
-    ACID_CUDA(cudaMemcpyAsync(p_prev, p_cur, sh.N * sh.d * sizeof(float), cudaMemcpyDeviceToDevice, s));
   } else {
     ACID_CUDA(cudaMemcpyAsync(w.x_prev, latent, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
     ACID_CUDA(cudaMemcpyAsync(v_prev, v, sh.latent * sizeof(float), cudaMemcpyDeviceToDevice, s));
@@ -931,17 +937,40 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
   return ACID_OK;
 }
 
-// One sampler step into `body`: the branch, the Euler update, the next step.
+// Sets the parity conditional of the step about to run (1: odd step).
+__global__ void parity_kernel(const DevLoop* st, cudaGraphConditionalHandle h_parity) {
+  cudaGraphSetConditional(h_parity, (unsigned)(st->step & 1));
+}
+
+// Opens the parity switch of a step in `body` (captured on gc.main): an
+// IF/ELSE node on the step's parity; returns its odd (bodies[0]) and even
+// (bodies[1]) graphs.
+acid_status capture_parity_switch(const LoopWs& w, GraphCapture& gc, cudaGraph_t body, cudaGraph_t* bodies) {
+  cudaGraphConditionalHandle h_parity;
+  ACID_CUDA(cudaGraphConditionalHandleCreate(&h_parity, body, 0, 0));
+  parity_kernel<<<1, 1, 0, gc.main>>>(w.dev, h_parity);
+  ACID_CHECK_LAUNCH();
+  return add_conditional(gc.main, h_parity, cudaGraphCondTypeIf, 2, bodies);
+}
+
+// One sampler step into `body`: the branch (one capture per parity, under the
+// parity switch), then the Euler update and the next step.
 acid_status capture_step(const acid_model& m, const acid_loop_cfg& cfg, LoopWs& w, float* latent, GraphCapture& gc,
                          cudaGraph_t body, cudaGraphConditionalHandle h_loop) {
   cudaStream_t s = gc.main;
+  cudaGraph_t tmp, pb[2];
   ACID_CUDA(cudaStreamBeginCaptureToGraph(s, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-  ACID_TRY(capture_branch(m, cfg, w, latent, gc, body));
+  ACID_TRY(capture_parity_switch(w, gc, body, pb));
   ACID_TRY(euler_update_sig(latent, w.v[0], shape_of(m).latent, w.sig, &w.dev->step, s));
   advance_kernel<<<1, 1, 0, s>>>(w.dev, nullptr, h_loop);
   ACID_CHECK_LAUNCH();
-  cudaGraph_t tmp;
   ACID_CUDA(cudaStreamEndCapture(s, &tmp));
+  for (int par = 0; par < 2; ++par) {
+    cudaGraph_t g = pb[par == 1 ? 0 : 1];
+    ACID_CUDA(cudaStreamBeginCaptureToGraph(s, g, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+    ACID_TRY(capture_branch(m, cfg, w, latent, gc, g, par));
+    ACID_CUDA(cudaStreamEndCapture(s, &tmp));
+  }
   return ACID_OK;
 }
 
@@ -950,14 +979,20 @@ acid_status capture_guided_step(const acid_model& m, const acid_loop_cfg& cc, co
                                 LoopWs& wc, LoopWs& wu, float* latent, GraphCapture& gc, cudaGraph_t body,
                                 cudaGraphConditionalHandle h_loop) {
   cudaStream_t s = gc.main;
+  cudaGraph_t tmp, pb[2];
   ACID_CUDA(cudaStreamBeginCaptureToGraph(s, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
-  ACID_TRY(capture_branch(m, cc, wc, latent, gc, body));
-  ACID_TRY(capture_branch(m, cu, wu, latent, gc, body));
+  ACID_TRY(capture_parity_switch(wc, gc, body, pb));
   ACID_TRY(guided_euler_update_sig(latent, wc.v[0], wu.v[0], shape_of(m).latent, scale, wc.sig, &wc.dev->step, s));
   advance_kernel<<<1, 1, 0, s>>>(wc.dev, wu.dev, h_loop);
   ACID_CHECK_LAUNCH();
-  cudaGraph_t tmp;
   ACID_CUDA(cudaStreamEndCapture(s, &tmp));
+  for (int par = 0; par < 2; ++par) {
+    cudaGraph_t g = pb[par == 1 ? 0 : 1];
+    ACID_CUDA(cudaStreamBeginCaptureToGraph(s, g, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed));
+    ACID_TRY(capture_branch(m, cc, wc, latent, gc, g, par));
+    ACID_TRY(capture_branch(m, cu, wu, latent, gc, g, par));
+    ACID_CUDA(cudaStreamEndCapture(s, &tmp));
+  }
   return ACID_OK;
 }
 

@@ -4,6 +4,7 @@ warm-up), for tuning and for profiler captures of a single launch.
     python -m paper_2607_12358_gb300.kernel_bench attention --n 32760 --heads 12 --head-dim 128
     python -m paper_2607_12358_gb300.kernel_bench linear --m 32760 --k 1536 --n 8960 --epi gelu
     python -m paper_2607_12358_gb300.kernel_bench drift --rows 118800 --cols 3072 [--apply]
+    python -m paper_2607_12358_gb300.kernel_bench temni --rows 32760 --cols 1536
     python -m paper_2607_12358_gb300.kernel_bench layernorm --rows 32760 --cols 1536 --in-dtype fp32
     python -m paper_2607_12358_gb300.kernel_bench block --workload wan [--block-type wan]
 
@@ -41,7 +42,7 @@ def _time(fn, warmup, iters):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("kernel", choices=["attention", "linear", "drift", "layernorm", "block"])
+    ap.add_argument("kernel", choices=["attention", "linear", "drift", "temni", "layernorm", "block"])
     ap.add_argument("--workload", default="wan", help="block: wan | cog | hv")
     ap.add_argument("--block-type", default=None, help="block: wan | cog | hv_dual | hv_single")
     ap.add_argument("--n", type=int, default=32760)
@@ -100,6 +101,19 @@ def main():
                    a.warmup, a.iters)
         nbytes = float(a.rows) * a.cols * (x.element_size() + 2)
         out.update(shape=[a.rows, a.cols], in_dtype=a.in_dtype, ms=ms, gbs=nbytes / ms / 1e6)
+    elif a.kernel == "temni":
+        # TeaCache signal from two steps' fp32 patch embeddings: reads 8 B/elem
+        hp = torch.randn(a.rows, a.cols, device=dev, generator=gen)
+        hc = hp + 0.05 * torch.randn(a.rows, a.cols, device=dev, generator=gen)
+        mp = 0.3 * torch.randn(2 * a.cols, device=dev, generator=gen)
+        mc = mp + 0.01 * torch.randn(2 * a.cols, device=dev, generator=gen)
+        ws = torch.empty(acid.drift_workspace_size(a.rows * a.cols), dtype=torch.uint8, device=dev)
+        rel = torch.empty(1, dtype=torch.float64, device=dev)
+        sums = torch.empty(2, dtype=torch.float64, device=dev)
+        ms = _time(lambda: acid.acid_temni_drift(hp, hc, mp, mc, out_rel=rel, out_sums=sums, workspace=ws),
+                   a.warmup, a.iters)
+        nbytes = 8.0 * a.rows * a.cols
+        out.update(shape=[a.rows, a.cols], ms=ms, gbs=nbytes / ms / 1e6, rel_l1=rel.item())
     elif a.kernel == "block":
         import acid_synth as S
 

@@ -179,3 +179,39 @@ def test_drift_and_apply_past_32_bit_offsets(acid):
     check_out(out)
     del prev, cur, res, out
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("rows,d", [(32760, 1536), (2049, 256), (777, 3072), (5, 1920), (1, 8)])
+def test_temni_drift_matches_oracle(acid, rows, d):
+    """acid_temni_drift: the TeaCache signal formed from two consecutive steps'
+    fp32 patch embeddings and block-0 modulations, against the oracle's
+    LayerNorm-modulate and relative L1 (Sec. 2, "TeaCache").  Shapes: the
+    Wan step's 32760 x 1536, row counts that leave partial groups of rows per
+    CTA, the widest rows (3072), a width that is not a multiple of 256, and
+    a single 8-wide row."""
+    rng = np.random.default_rng(rows + d)
+    h_prev = rng.normal(size=(rows, d)).astype(np.float32)
+    h_cur = (h_prev + 0.05 * rng.normal(size=(rows, d))).astype(np.float32)
+    mod_prev = (0.3 * rng.normal(size=2 * d)).astype(np.float32)
+    mod_cur = (mod_prev + 0.01 * rng.normal(size=2 * d)).astype(np.float32)
+    t = {k: torch.from_numpy(v).to(DEV) for k, v in (("hp", h_prev), ("hc", h_cur), ("mp", mod_prev), ("mc", mod_cur))}
+    rel, sums = acid.acid_temni_drift(t["hp"], t["hc"], t["mp"], t["mc"], eps=1e-6)
+    torch.cuda.synchronize()
+    acid.check_device_error()
+    up = O.modulate(O.layer_norm(h_prev, 1e-6), mod_prev[:d], mod_prev[d:])
+    uc = O.modulate(O.layer_norm(h_cur, 1e-6), mod_cur[:d], mod_cur[d:])
+    ref = O.rel_l1(up, uc)
+    assert abs(rel.item() - ref) <= DRIFT_RTOL * ref, (rel.item(), ref)
+    np.testing.assert_allclose(sums.cpu().numpy(), [np.abs(uc - up).sum(), np.abs(up).sum()], rtol=DRIFT_RTOL)
+
+
+def test_temni_drift_identical_steps_and_empty(acid):
+    """The same h and modulation on both steps give exactly 0; zero rows give 0."""
+    rng = np.random.default_rng(5)
+    h = torch.from_numpy(rng.normal(size=(300, 1536)).astype(np.float32)).to(DEV)
+    m = torch.from_numpy((0.2 * rng.normal(size=3072)).astype(np.float32)).to(DEV)
+    rel, sums = acid.acid_temni_drift(h, h, m, m)
+    assert rel.item() == 0.0 and sums[0].item() == 0.0 and sums[1].item() > 0
+    e = torch.empty((0, 1536), dtype=torch.float32, device=DEV)
+    rel, sums = acid.acid_temni_drift(e, e, m, m)
+    assert rel.item() == 0.0 and sums.cpu().tolist() == [0.0, 0.0]

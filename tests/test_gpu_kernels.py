@@ -126,6 +126,32 @@ def test_linear_bf16_partial_last_column_tile(acid, M, K, N, epi):
     assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
 
 
+@pytest.mark.parametrize("M,K,N", [(891, 2112, 1024), (130, 4160, 2304), (1000, 64, 4096), (257, 2176, 160)])
+@pytest.mark.parametrize("epi,fp32", [("bias", True), ("gelu", False), ("gated_res", True), ("res", False)])
+def test_linear_bf16_pair_tiles(acid, M, K, N, epi, fp32):
+    """Shapes that run on SM pairs (N or K above 2048): 256-row pair tiles
+    whose second CTA holds a ragged (123, 2) or a full last row block, a K
+    that is a multiple of 64 with many stage-ring wraps, N a multiple of 256,
+    and a 160-wide output whose second CTA's weight rows lie beyond N."""
+    rng = np.random.default_rng(M + 3 * K + 5 * N)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.05 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    g = rng.normal(size=N).astype(np.float32)
+    r = rng.normal(size=(M, N)).astype(np.float32)
+    if not fp32:
+        r = S.round_to_bf16(r)
+    has_res = epi in ("gated_res", "res")
+    res = (_f32(r) if fp32 else _bf(r)) if has_res else None
+    out = acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), epilogue=epi, gate=_f32(g), residual=res, out=res,
+                                   out_fp32=fp32)
+    acc = O.linear(a, w, b)
+    ref = {"bias": acc, "gelu": O.gelu_tanh(acc), "gated_res": r + g * acc, "res": r + acc}[epi]
+    got = out.float().cpu().numpy()
+    tol = 1e-4 if (fp32 and epi != "gelu") else 2 ** -8
+    assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
+
+
 def test_linear_bf16_offsets_past_32_bits(acid):
     """An output of 262181 x 8960 fp32 values (2.35e9 elements, 9.4 GB),
     updated in place by the gated-residual epilogue.  Rows from 239675 on
