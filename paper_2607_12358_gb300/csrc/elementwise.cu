@@ -336,15 +336,6 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
   uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)nwarps * kTemniStages * 2 * d);  // [warp][stage]
   __shared__ double rd[2][kTemniMaxWarps];
   const int step = step_dev ? *step_dev : step_host;
-  for (int i = threadIdx.x; i < d / 4; i += blockDim.x) {
-    const float4 a = reinterpret_cast<const float4*>(shc)[i], b = reinterpret_cast<const float4*>(scc)[i];
-    const float4 c = reinterpret_cast<const float4*>(shp)[i], e = reinterpret_cast<const float4*>(scp)[i];
-    const int q = d / 4;
-    mod[i] = a;
-    mod[q + i] = make_float4(1.f + b.x, 1.f + b.y, 1.f + b.z, 1.f + b.w);
-    mod[2 * q + i] = c;
-    mod[3 * q + i] = make_float4(1.f + e.x, 1.f + e.y, 1.f + e.z, 1.f + e.w);
-  }
   float* wr = ring + (size_t)warp * kTemniStages * 2 * d;
   uint64_t* wf = full + warp * kTemniStages;
   const int64_t gw = (int64_t)blockIdx.x * nwarps + warp, nw = (int64_t)gridDim.x * nwarps;
@@ -357,10 +348,21 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
     bulk_load(wr + (size_t)st * 2 * d, xc + row * d, row_bytes, &wf[st]);
     bulk_load(wr + (size_t)st * 2 * d + d, xp + row * d, row_bytes, &wf[st]);
   };
+  // each warp's first copies are issued before the modulation vectors are
+  // staged, so their latency overlaps the staging
   if (lane == 0) {
     for (int i = 0; i < kTemniStages; ++i) mbar_init(&wf[i], 1);
     mbar_fence_init();
     for (int64_t k = 0; k < n_my && k < kTemniStages; ++k) issue(k);
+  }
+  for (int i = threadIdx.x; i < d / 4; i += blockDim.x) {
+    const float4 a = reinterpret_cast<const float4*>(shc)[i], b = reinterpret_cast<const float4*>(scc)[i];
+    const float4 c = reinterpret_cast<const float4*>(shp)[i], e = reinterpret_cast<const float4*>(scp)[i];
+    const int q = d / 4;
+    mod[i] = a;
+    mod[q + i] = make_float4(1.f + b.x, 1.f + b.y, 1.f + b.z, 1.f + b.w);
+    mod[2 * q + i] = c;
+    mod[3 * q + i] = make_float4(1.f + e.x, 1.f + e.y, 1.f + e.z, 1.f + e.w);
   }
   __syncthreads();  // modulation vectors staged, barriers initialised
   const float inv_d = 1.0f / d;

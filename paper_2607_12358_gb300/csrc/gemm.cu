@@ -243,9 +243,41 @@ __device__ __forceinline__ float4* stage_unit(float* stage, int row, int unit) {
   return reinterpret_cast<float4*>(stage) + row * 8 + (unit ^ (row & 7));
 }
 
-template <int KIND, bool R32>
-__device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, float* stage, int64_t row0,
-                                               int col0, const uint32_t* r, const ResChunk<R32>& rc) {
+// Output box of one chunk in the stage, as the tensor store reads it: 32 rows
+// x 32 columns, row-major.  fp32: 128-byte rows with the 128-byte swizzle
+// (16-byte unit u of row r at u ^ (r & 7)), the stage's own layout, so each
+// lane overwrites in place the 16 bytes it has just read.  bf16: 64-byte rows
+// with the 64-byte swizzle (unit u at u ^ ((r >> 1) & 3)); box row r lies in
+// stage row r / 2, which the warp has read by the time row group r / 4 is
+// written (row groups are written behind a __syncwarp).
+__device__ __forceinline__ void box_store_f32(float* stage, int rr, int lane, const float* v) {
+  *stage_unit(stage, rr, lane & 7) = make_float4(v[0], v[1], v[2], v[3]);
+}
+__device__ __forceinline__ void box_store_bf16(float* stage, int rr, int lane, const float* v) {
+  const int u = (lane & 7) >> 1;
+  uint8_t* p = reinterpret_cast<uint8_t*>(stage) + rr * 64 + ((u ^ ((rr >> 1) & 3)) << 4) + (lane & 1) * 8;
+  *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
+}
+
+// Output stores of the epilogue: kinds without a residual write each chunk's
+// results back into the stage as the output box and hand it to one tensor
+// store (the TMA engine then writes the 2-4 KB box; rows past M and columns
+// past N are clipped by the tensor map).  The residual kinds keep a residual
+// prefetch of two chunks in registers and store directly from registers
+// (coalesced 8-16-byte stores per lane), which leaves them without spills at
+// the 168-register limit of ten warps.
+template <int KIND>
+constexpr bool kTmaStore = !(KIND == EPI_GATED_RES || KIND == EPI_RES);
+
+// Epilogue of one 32-row x 32-column chunk held by a warp (thread = row, as
+// tcgen05.ld delivers it).  The chunk is transposed through the stage so that
+// each lane handles four columns of eight rows, then stored as above.  With
+// tensor stores the caller waits for the previous store to have read the
+// stage before calling again.
+template <int KIND, bool R32, bool O32>
+__device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& e, const CUtensorMap* tmO,
+                                               float* stage, int64_t row0, int col0, const uint32_t* r,
+                                               const ResChunk<R32>& rc) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
   for (int u = 0; u < 8; ++u)
@@ -255,8 +287,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
   const int c = 4 * (lane & 7);
   const int col = col0 + c;
   // RoPE: the (cos, sin) of this lane's two pairs on its eight rows, all
-  // loaded through the read-only path before any output is stored, so that
-  // the loads overlap instead of queueing behind the stores
+  // loaded through the read-only path before the row groups are processed
   float2 rcs[KIND == EPI_ROPE_QKV ? 8 : 1][2];
   if constexpr (KIND == EPI_ROPE_QKV) {
     const int j0 = (col & (e.head_dim - 1)) >> 1;
@@ -273,13 +304,11 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
   }
   const uint64_t b01 = f2_pack(rc.bias[0], rc.bias[1]), b23 = f2_pack(rc.bias[2], rc.bias[3]);
   // rows past M are computed like the others (from whatever the stage and
-  // residual registers hold) and only their stores are skipped, so the eight
-  // row groups form one branch-free block the compiler can interleave
+  // residual registers hold); the tensor store clips them
 #pragma unroll
   for (int p = 0; p < 8; ++p) {
     const int rr = 4 * p + (lane >> 3);
-    const int64_t row = row0 + rr;
-    const int64_t grow = row + e.row_base;
+    const int64_t grow = row0 + rr + e.row_base;
     const float4 sv = *stage_unit(stage, rr, lane & 7);
     uint64_t v01 = f2_add(f2_pack(sv.x, sv.y), b01), v23 = f2_add(f2_pack(sv.z, sv.w), b23);
     switch (KIND) {
@@ -322,20 +351,39 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
     float v[4];
     f2_unpack(v01, v[0], v[1]);
     f2_unpack(v23, v[2], v[3]);
-    if (row >= g.M) continue;
-    if (g.out_fp32)
-      *reinterpret_cast<float4*>(static_cast<float*>(g.out) + row * g.ldo + col) = make_float4(v[0], v[1], v[2], v[3]);
-    else
-      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col) =
-          make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
+    if constexpr (kTmaStore<KIND>) {
+      if constexpr (O32) {
+        box_store_f32(stage, rr, lane, v);  // in place: this lane's own 16 bytes
+      } else {
+        __syncwarp();  // the stage row this box row overwrites has been read by every lane
+        box_store_bf16(stage, rr, lane, v);
+      }
+    } else {
+      const int64_t row = row0 + rr;
+      if (row >= g.M) continue;
+      if constexpr (O32)
+        *reinterpret_cast<float4*>(static_cast<float*>(g.out) + row * g.ldo + col) = make_float4(v[0], v[1], v[2], v[3]);
+      else
+        *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(g.out) + row * g.ldo + col) =
+            make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
+    }
   }
-  __syncwarp();
+  if constexpr (kTmaStore<KIND>) {
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tmO, stage, col0, (int)row0);
+      bulk_commit_group();
+    }
+  } else {
+    __syncwarp();  // every lane has read the stage before the next chunk overwrites it
+  }
 }
 
-template <int BN, int KIND, bool R32>
+template <int BN, int KIND, bool R32, bool O32>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
-                   EpiDev e) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmO, GemmDims g, EpiDev e) {
   using C = TcCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -450,7 +498,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         tmem_wait_ld();
         const int col0 = n_tile * BN + c;
         if (i + 1 < NC && row0 < g.M && col0 + 32 < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, col0 + 32 + lcol, nxt);
-        if (ok && row0 < g.M && col0 < g.N) epilogue_chunk<KIND, R32>(g, e, stage, row0, col0, r, cur);
+        if (ok && row0 < g.M && col0 < g.N) {
+          if constexpr (kTmaStore<KIND>) {
+            if (lane == 0) bulk_wait_group_read<0>();  // the previous box has left the stage
+            __syncwarp();
+          }
+          epilogue_chunk<KIND, R32, O32>(g, e, &tmO, stage, row0, col0, r, cur);
+        }
       };
       ResChunk<R32> rc0, rc1;
       if (row0 < g.M && n_tile * BN + cbeg < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, n_tile * BN + cbeg + lcol, rc0);
@@ -463,6 +517,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_arrive(&acc_empty[b]);
       if (!ok) break;
     }
+    if (lane == 0) bulk_wait_group<0>();  // tensor stores complete before the CTA exits
   }
   tc_fence_before();
   __syncthreads();
@@ -504,10 +559,10 @@ struct Tc2Cfg {
 };
 static_assert(Tc2Cfg::SMEM <= 232448, "pair GEMM shared memory");
 
-template <int KIND, bool R32>
+template <int KIND, bool R32, bool O32>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
-    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, GemmDims g,
-                    EpiDev e) {
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmO, GemmDims g, EpiDev e) {
   using C = Tc2Cfg;
   constexpr int BN = C::BN;
   extern __shared__ uint8_t smem_raw[];
@@ -637,7 +692,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         tmem_wait_ld();
         const int col0 = n_tile * BN + c;
         if (i + 1 < NC && row0 < g.M && col0 + 32 < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, col0 + 32 + lcol, nxt);
-        if (ok && row0 < g.M && col0 < g.N) epilogue_chunk<KIND, R32>(g, e, stage, row0, col0, r, cur);
+        if (ok && row0 < g.M && col0 < g.N) {
+          if constexpr (kTmaStore<KIND>) {
+            if (lane == 0) bulk_wait_group_read<0>();  // the previous box has left the stage
+            __syncwarp();
+          }
+          epilogue_chunk<KIND, R32, O32>(g, e, &tmO, stage, row0, col0, r, cur);
+        }
       };
       ResChunk<R32> rc0, rc1;
       if (row0 < g.M && n_tile * BN + cbeg < g.N) load_chunk_inputs<KIND, R32>(g, e, row0, n_tile * BN + cbeg + lcol, rc0);
@@ -651,6 +712,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       if (lane == 0) mbar_arrive_cluster(acc_empty0 + 8 * b);
       if (!ok) break;
     }
+    if (lane == 0) bulk_wait_group<0>();  // tensor stores complete before the CTA exits
   }
   tc_fence_before();
   __syncthreads();
@@ -680,23 +742,28 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 }  // namespace
 
-// Row-major bf16 matrix [rows, cols] with row stride ld (elements), boxes of
-// box_rows x box_cols, the given swizzle, zero fill out of bounds.
-acid_status make_tmap_bf16_box(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
-                               int box_cols, int box_rows, CUtensorMapSwizzle swizzle) {
+// Row-major matrix [rows, cols] of 2-byte (bf16) or 4-byte (fp32) elements
+// with row stride ld (elements), boxes of box_rows x box_cols, the given
+// swizzle, zero fill out of bounds (loads) and clipping (stores).
+acid_status make_tmap_2d(CUtensorMap* map, CUtensorMapDataType type, int esize, const void* base, int64_t rows,
+                         int64_t cols, int64_t ld, int box_cols, int box_rows, CUtensorMapSwizzle swizzle) {
   auto fn = encode_fn();
   ACID_REQUIRE(fn != nullptr, ACID_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
-  ACID_REQUIRE(aligned(base, 16) && (ld * 2) % 16 == 0, ACID_ERR_UNSUPPORTED,
-               "TMA operand must be 16-byte aligned with a row stride that is a multiple of 8 elements");
+  ACID_REQUIRE(aligned(base, 16) && (ld * esize) % 16 == 0, ACID_ERR_UNSUPPORTED,
+               "TMA operand must be 16-byte aligned with a row stride that is a multiple of 16 bytes");
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * esize)};
   cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1u, 1u};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(map, type, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   ACID_REQUIRE(r == CUDA_SUCCESS, ACID_ERR_CUDA, "cuTensorMapEncodeTiled failed (code " + std::to_string((int)r) + ")");
   return ACID_OK;
+}
+
+acid_status make_tmap_bf16_box(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                               int box_cols, int box_rows, CUtensorMapSwizzle swizzle) {
+  return make_tmap_2d(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, rows, cols, ld, box_cols, box_rows, swizzle);
 }
 
 // Boxes of box_rows x 64 columns with 128-byte swizzle (the MMA operand layout).
@@ -705,6 +772,14 @@ acid_status make_tmap_bf16(CUtensorMap* map, const void* base, int64_t rows, int
 }
 
 namespace {
+
+// The GEMM output as the epilogue's tensor stores see it: 32 x 32 boxes, the
+// swizzle of the box layout in epilogue_chunk (128-byte rows for fp32,
+// 64-byte rows for bf16).
+acid_status make_tmap_out(CUtensorMap* map, void* out, int64_t M, int N, int64_t ldo, bool fp32) {
+  return fp32 ? make_tmap_2d(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, out, M, N, ldo, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B)
+              : make_tmap_2d(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, out, M, N, ldo, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+}
 
 int num_sms() {
   static int n = 0;
@@ -716,46 +791,55 @@ int num_sms() {
   return n;
 }
 
-template <int BN, int KIND, bool R32 = false>
-acid_status launch_tc_kind(const CUtensorMap& ta, const CUtensorMap& tb, const GemmDims& g, const Epilogue& epi,
-                           int grid, cudaStream_t s) {
+template <int BN, int KIND, bool R32, bool O32>
+acid_status launch_tc_kind1(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& to, const GemmDims& g,
+                           const Epilogue& epi, int grid, cudaStream_t s) {
   using C = TcCfg<BN>;
   static bool attr_done = false;
   if (!attr_done) {
-    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN, KIND, R32>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
+    ACID_CUDA(cudaFuncSetAttribute(gemm_tc_kernel<BN, KIND, R32, O32>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM));
     attr_done = true;
   }
-  gemm_tc_kernel<BN, KIND, R32><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, g, to_dev(epi));
+  gemm_tc_kernel<BN, KIND, R32, O32><<<grid, kGemmThreads, C::SMEM, s>>>(ta, tb, to, g, to_dev(epi));
   ACID_CHECK_LAUNCH();
   return ACID_OK;
+}
+
+// dispatch on the output dtype (a template parameter: it selects the box layout)
+template <int BN, int KIND, bool R32 = false>
+acid_status launch_tc_kind(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& to, const GemmDims& g,
+                           const Epilogue& epi, int grid, cudaStream_t s) {
+  return g.out_fp32 ? launch_tc_kind1<BN, KIND, R32, true>(ta, tb, to, g, epi, grid, s)
+                    : launch_tc_kind1<BN, KIND, R32, false>(ta, tb, to, g, epi, grid, s);
 }
 
 template <int BN>
 acid_status launch_tc(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
                       const Epilogue& epi, cudaStream_t s) {
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, to;
   ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
   ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, BN));
+  ACID_TRY(make_tmap_out(&to, out, M, N, ldo, epi.out_fp32));
   GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0};
   const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = (int)std::min<int64_t>(tiles, num_sms());
   ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
   switch (epi.kind) {
-    case EPI_GELU: return launch_tc_kind<BN, EPI_GELU>(ta, tb, g, epi, grid, s);
-    case EPI_ROPE_QKV: return launch_tc_kind<BN, EPI_ROPE_QKV>(ta, tb, g, epi, grid, s);
+    case EPI_GELU: return launch_tc_kind<BN, EPI_GELU>(ta, tb, to, g, epi, grid, s);
+    case EPI_ROPE_QKV: return launch_tc_kind<BN, EPI_ROPE_QKV>(ta, tb, to, g, epi, grid, s);
     case EPI_GATED_RES:
-      return epi.res_fp32 ? launch_tc_kind<BN, EPI_GATED_RES, true>(ta, tb, g, epi, grid, s)
-                          : launch_tc_kind<BN, EPI_GATED_RES, false>(ta, tb, g, epi, grid, s);
+      return epi.res_fp32 ? launch_tc_kind<BN, EPI_GATED_RES, true>(ta, tb, to, g, epi, grid, s)
+                          : launch_tc_kind<BN, EPI_GATED_RES, false>(ta, tb, to, g, epi, grid, s);
     case EPI_RES:
-      return epi.res_fp32 ? launch_tc_kind<BN, EPI_RES, true>(ta, tb, g, epi, grid, s)
-                          : launch_tc_kind<BN, EPI_RES, false>(ta, tb, g, epi, grid, s);
-    default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, g, epi, grid, s);
+      return epi.res_fp32 ? launch_tc_kind<BN, EPI_RES, true>(ta, tb, to, g, epi, grid, s)
+                          : launch_tc_kind<BN, EPI_RES, false>(ta, tb, to, g, epi, grid, s);
+    default: return launch_tc_kind<BN, EPI_BIAS>(ta, tb, to, g, epi, grid, s);
   }
 }
 
 // CTA pairs that can be resident at once for the pair kernel (clusters are
 // placed within a GPC, so this can be below half the SM count).
-template <int KIND, bool R32>
+template <int KIND, bool R32, bool O32>
 int max_pairs() {
   static int n = -1;
   if (n < 0) {
@@ -764,46 +848,54 @@ int max_pairs() {
     cfg.blockDim = dim3(kGemmThreads, 1, 1);
     cfg.dynamicSmemBytes = Tc2Cfg::SMEM;
     int c = 0;
-    n = (cudaOccupancyMaxActiveClusters(&c, gemm_tc2_kernel<KIND, R32>, &cfg) == cudaSuccess && c > 0) ? c : 0;
+    n = (cudaOccupancyMaxActiveClusters(&c, gemm_tc2_kernel<KIND, R32, O32>, &cfg) == cudaSuccess && c > 0) ? c : 0;
   }
   return n;
 }
 
-template <int KIND, bool R32 = false>
-acid_status launch_tc2_kind(const CUtensorMap& ta, const CUtensorMap& tb, const GemmDims& g, const Epilogue& epi,
-                            int64_t tiles, cudaStream_t s) {
+template <int KIND, bool R32, bool O32>
+acid_status launch_tc2_kind1(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& to, const GemmDims& g,
+                            const Epilogue& epi, int64_t tiles, cudaStream_t s) {
   static bool attr_done = false;
   if (!attr_done) {
-    ACID_CUDA(cudaFuncSetAttribute(gemm_tc2_kernel<KIND, R32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    ACID_CUDA(cudaFuncSetAttribute(gemm_tc2_kernel<KIND, R32, O32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    Tc2Cfg::SMEM));
     attr_done = true;
   }
-  const int pairs = max_pairs<KIND, R32>();
+  const int pairs = max_pairs<KIND, R32, O32>();
   ACID_REQUIRE(pairs > 0, ACID_ERR_CUDA, "linear: no resident CTA pair for the pair GEMM");
   const int grid = 2 * (int)std::min<int64_t>(tiles, pairs);
-  gemm_tc2_kernel<KIND, R32><<<grid, kGemmThreads, Tc2Cfg::SMEM, s>>>(ta, tb, g, to_dev(epi));
+  gemm_tc2_kernel<KIND, R32, O32><<<grid, kGemmThreads, Tc2Cfg::SMEM, s>>>(ta, tb, to, g, to_dev(epi));
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }
 
+template <int KIND, bool R32 = false>
+acid_status launch_tc2_kind(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& to, const GemmDims& g,
+                            const Epilogue& epi, int64_t tiles, cudaStream_t s) {
+  return g.out_fp32 ? launch_tc2_kind1<KIND, R32, true>(ta, tb, to, g, epi, tiles, s)
+                    : launch_tc2_kind1<KIND, R32, false>(ta, tb, to, g, epi, tiles, s);
+}
+
 acid_status launch_tc2(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out, int64_t ldo,
                        const Epilogue& epi, cudaStream_t s) {
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, to;
   ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
   ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, Tc2Cfg::BN / 2));
+  ACID_TRY(make_tmap_out(&to, out, M, N, ldo, epi.out_fp32));
   GemmDims g{M, N, K, out, ldo, epi.out_fp32 ? 1 : 0};
   const int64_t tiles = ((M + 2 * BM - 1) / (2 * BM)) * ((N + Tc2Cfg::BN - 1) / Tc2Cfg::BN);
   ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
   switch (epi.kind) {
-    case EPI_GELU: return launch_tc2_kind<EPI_GELU>(ta, tb, g, epi, tiles, s);
-    case EPI_ROPE_QKV: return launch_tc2_kind<EPI_ROPE_QKV>(ta, tb, g, epi, tiles, s);
+    case EPI_GELU: return launch_tc2_kind<EPI_GELU>(ta, tb, to, g, epi, tiles, s);
+    case EPI_ROPE_QKV: return launch_tc2_kind<EPI_ROPE_QKV>(ta, tb, to, g, epi, tiles, s);
     case EPI_GATED_RES:
-      return epi.res_fp32 ? launch_tc2_kind<EPI_GATED_RES, true>(ta, tb, g, epi, tiles, s)
-                          : launch_tc2_kind<EPI_GATED_RES, false>(ta, tb, g, epi, tiles, s);
+      return epi.res_fp32 ? launch_tc2_kind<EPI_GATED_RES, true>(ta, tb, to, g, epi, tiles, s)
+                          : launch_tc2_kind<EPI_GATED_RES, false>(ta, tb, to, g, epi, tiles, s);
     case EPI_RES:
-      return epi.res_fp32 ? launch_tc2_kind<EPI_RES, true>(ta, tb, g, epi, tiles, s)
-                          : launch_tc2_kind<EPI_RES, false>(ta, tb, g, epi, tiles, s);
-    default: return launch_tc2_kind<EPI_BIAS>(ta, tb, g, epi, tiles, s);
+      return epi.res_fp32 ? launch_tc2_kind<EPI_RES, true>(ta, tb, to, g, epi, tiles, s)
+                          : launch_tc2_kind<EPI_RES, false>(ta, tb, to, g, epi, tiles, s);
+    default: return launch_tc2_kind<EPI_BIAS>(ta, tb, to, g, epi, tiles, s);
   }
 }
 
