@@ -234,6 +234,21 @@ __device__ __forceinline__ void load_kv_tile(uint8_t* dst, const CUtensorMap* ma
   for (int c = 0; c < C::CH; ++c) tma_load_2d(dst + c * C::CHUNK_KV, map, bar, col + c * 64, row);
 }
 
+// Failure path (a wait ran out): the producer waits, bounded, until the loads
+// it has issued have landed (the Q tiles, and the last K and V tiles of each
+// two-slot ring), so that no copy writes into the shared memory of a CTA
+// that has left; the MMA thread waits, bounded, for the MMAs it has issued
+// before tensor memory is freed.  Never called on the normal path.
+__device__ __noinline__ void drain_loads(uint64_t* q_full, uint64_t* k_full, uint64_t* v_full, int nk, int nv) {
+  mbar_wait(q_full, 0);
+  for (int j = nk > 2 ? nk - 2 : 0; j < nk; ++j) mbar_wait(&k_full[j & 1], (j >> 1) & 1);
+  for (int j = nv > 2 ? nv - 2 : 0; j < nv; ++j) mbar_wait(&v_full[j & 1], (j >> 1) & 1);
+}
+__device__ __noinline__ void drain_mmas(uint64_t* drain) {
+  mma_commit(drain);
+  mbar_wait(drain, 0);
+}
+
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -253,6 +268,7 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
   uint64_t* s_full = bars + 9;    // [2] per query tile
   uint64_t* p_full = bars + 11;   // [2] per query tile
   uint64_t* pv_done = bars + 13;  // [2] per query tile
+  uint64_t* drain = bars + 15;    // failure path: the MMAs issued so far have completed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -276,6 +292,7 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
       mbar_init(&p_full[i], 128);
       mbar_init(&pv_done[i], 1);
     }
+    mbar_init(drain, 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -291,13 +308,17 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
         for (int c = 0; c < C::CH; ++c)
           tma_load_2d(sQ + t * C::T_BYTES + c * C::CHUNK_Q, &tmQ, q_full, a.q_col + h * D + c * 64,
                       qt * kBQ + t * kTileQ);
+      int nk_issued = 0, nv_issued = 0;
       for (int j = 0; j < nkv; ++j) {
         const int st = j & 1, round = j >> 1;
         if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) break;
         load_kv_tile<D>(sK + st * C::KV_BYTES, &tmK, &k_full[st], a.k_col + h * D, (jb + j) * C::BKV);
+        nk_issued = j + 1;
         if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) break;
         load_kv_tile<D>(sV + st * C::KV_BYTES, &tmV, &v_full[st], a.v_col + h * D, (jb + j) * C::BKV);
+        nv_issued = j + 1;
       }
+      if (nv_issued < nkv) drain_loads(q_full, k_full, v_full, nk_issued, nv_issued);
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------------------------------- MMA issuer
@@ -339,6 +360,7 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
           }
         }
       }
+      if (!ok) drain_mmas(drain);
     }
   } else {  // ---------------------------------------- softmax: warps 2-5 tile a, 6-9 tile b
     const int t = (warp - 2) >> 2;
@@ -431,7 +453,8 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
   uint64_t* s_full = bars + 12;   // [2] per query tile
   uint64_t* p_full = bars + 14;   // [2] per query tile
   uint64_t* pv_done = bars + 16;  // [2] per query tile
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  uint64_t* drain = bars + 18;    // failure path: the MMAs issued so far have completed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 19);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int item0 = a.item_base + (int)blockIdx.x, item_step = (int)gridDim.x;
@@ -455,6 +478,7 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
       mbar_init(&p_full[i], 128);
       mbar_init(&pv_done[i], 1);
     }
+    mbar_init(drain, 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -466,6 +490,7 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
   if (warp == 0) {
     if (lane == 0) {  // ---------------------------------------- TMA producer
       bool ok = true;
+      int nk_issued = 0, nv_issued = 0;
       for (int k = 0, g = 0; ok && k < n_items; ++k) {
         const int item = item0 + k * item_step;
         const int qt = item % a.nqp, h = item / a.nqp;
@@ -481,9 +506,17 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
           const int st = g & 1, round = g >> 1;
           if (round > 0 && !mbar_wait(&k_empty[st], (round - 1) & 1)) { ok = false; break; }
           load_kv_tile<D>(sK + st * C::KV_BYTES, &tmK, &k_full[st], a.k_col + h * D, j * C::BKV);
+          nk_issued = g + 1;
           if (round > 0 && !mbar_wait(&v_empty[st], (round - 1) & 1)) { ok = false; break; }
           load_kv_tile<D>(sV + st * C::KV_BYTES, &tmV, &v_full[st], a.v_col + h * D, j * C::BKV);
+          nv_issued = g + 1;
         }
+      }
+      // after a wait ran out: the last K and V loads of each ring have landed
+      // (Q loads of an item are waited on by the MMA thread before any use)
+      if (!ok) {
+        for (int j = nk_issued > 2 ? nk_issued - 2 : 0; j < nk_issued; ++j) mbar_wait(&k_full[j & 1], (j >> 1) & 1);
+        for (int j = nv_issued > 2 ? nv_issued - 2 : 0; j < nv_issued; ++j) mbar_wait(&v_full[j & 1], (j >> 1) & 1);
       }
     }
   } else if (warp == 1) {
@@ -531,6 +564,7 @@ __global__ void __launch_bounds__(kAttnThreads, AttnCfg<D>::CTAS_PER_SM)
         j = jn;
         k += boundary;
       }
+      if (!ok) drain_mmas(drain);
     }
   } else {  // ---------------------------------------- softmax: warps 2-5 tile a, 6-9 tile b
     const int t = (warp - 2) >> 2;
