@@ -44,9 +44,10 @@ MICRO_SIGMA = 1e-2
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, ncu captures of
 # a self-attention call (main launch, split tail launch and merge) and a
 # cross-attention call (one persistent launch) at this shape, each the mean of
-# two calls) per attention call of the step's 1:1 self/cross mix.  Valid only for the kernel source it was measured on; any
-# other source reports null.
-ATTN_TRAFFIC = {"source_sha256_16": "f4686df233990ff3", "bytes_per_launch": (435.47e6 + 159.20e6) / 2}
+# two calls) per attention call of the step's 1:1 self/cross mix: 436.9 MB and
+# 159.2 MB.  Valid only for the kernel source it was measured on; any other
+# source reports null.
+ATTN_TRAFFIC = {"source_sha256_16": "c918258b40c85349", "bytes_per_launch": (436.88e6 + 159.20e6) / 2}
 
 
 def _attn_traffic():

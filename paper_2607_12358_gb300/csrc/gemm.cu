@@ -955,11 +955,8 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__
       }
       float a = acc[i][j], b = acc[i][j + 1];
       epi_pair<false>(e, grow, col, a, b, r0, r1);
-      // evict-first: the patch embedding's 201 MB output at the Wan shape
-      // would otherwise sit in L2 as dirty lines, and their write-back
-      // would fall into the next kernel (the drift) instead of this one
-      __stcs(&out[row * ldo + col], a);
-      __stcs(&out[row * ldo + col + 1], b);
+      out[row * ldo + col] = a;
+      out[row * ldo + col + 1] = b;
     }
   }
 }
