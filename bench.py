@@ -311,6 +311,26 @@ def micro_bench(acid, dev, peaks: dict, iters: int = 20) -> dict:
         del p, c, r, o, ws
     out["min_frac_of_hbm"] = worst
     out["hbm_peak"] = hbm
+    # the TeaCache signal from two steps' fp32 patch embeddings
+    # (acid_temni_drift: reads 8 B/elem, the call includes the final
+    # reduction), at the Wan step's shape and at a 720p-class row count
+    out["temni"] = {}
+    for rows, d in ((32760, 1536), (118800, 1536)):
+        hp = torch.randn(rows, d, device=dev, generator=gen)
+        hc = hp + 0.05 * torch.randn(rows, d, device=dev, generator=gen)
+        mp = 0.3 * torch.randn(2 * d, device=dev, generator=gen)
+        mc = mp + 0.01 * torch.randn(2 * d, device=dev, generator=gen)
+        ws = torch.empty(acid.drift_workspace_size(rows * d), dtype=torch.uint8, device=dev)
+        rel = torch.empty(1, dtype=torch.float64, device=dev)
+        sums = torch.empty(2, dtype=torch.float64, device=dev)
+        fn = lambda: acid.acid_temni_drift(hp, hc, mp, mc, out_rel=rel, out_sums=sums, workspace=ws)
+        fn()
+        fn()
+        ms = _launch_ms(fn, iters)
+        gbs = 8.0 * rows * d / ms / 1e6
+        out["temni"][f"{rows}x{d}"] = {"ms": ms, "gbs": gbs, "frac_of_hbm": gbs / hbm, "bytes_per_elem": 8.0,
+                                       "kernel": "temni_drift_kernel + drift_final_kernel"}
+        del hp, hc, ws
     torch.cuda.empty_cache()
     return out
 
