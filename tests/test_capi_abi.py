@@ -123,6 +123,20 @@ def test_host_validation_without_gpu(lib):
                                        None, None, 0, 0, None) == want
     n = ctypes.c_size_t()
     assert lib.acid_attention_workspace_size(128, ctypes.byref(n)) == A.ACID_OK and n.value > 0
+    # TEMNI drift: shapes, pointers, alignment and workspace are checked before
+    # any device work (the pointer values below are never dereferenced)
+    f = lib.acid_temni_drift
+    out = ctypes.c_double()
+    po = ctypes.byref(out)
+    assert f(None, None, None, None, 10, 1004, 1e-6, po, None, None, 0, None) == A.ACID_ERR_UNSUPPORTED  # d % 8
+    assert f(None, None, None, None, 10, 4096, 1e-6, po, None, None, 0, None) == A.ACID_ERR_UNSUPPORTED  # d > 3072
+    assert f(None, None, None, None, -1, 1536, 1e-6, po, None, None, 0, None) == A.ACID_ERR_INVALID_ARG
+    assert f(None, None, None, None, 10, 1536, 1e-6, None, None, None, 0, None) == A.ACID_ERR_INVALID_ARG
+    assert f(None, None, None, None, 10, 1536, 1e-6, po, None, None, 0, None) == A.ACID_ERR_INVALID_ARG
+    assert f(8, 16, 16, 16, 10, 1536, 1e-6, po, None, 256, 1 << 20, None) == A.ACID_ERR_UNSUPPORTED  # misaligned
+    assert f(16, 16, 16, 16, 10, 1536, 1e-6, po, None, None, 0, None) == A.ACID_ERR_WORKSPACE
+    assert f(16, 16, 16, 16, 10, 1536, 1e-6, po, None, 256, 100, None) == A.ACID_ERR_WORKSPACE
+    assert b"workspace too small" in lib.acid_last_error()
 
 
 def test_loop_workspace_size_without_gpu(lib):
