@@ -138,6 +138,17 @@ __global__ void __launch_bounds__(kThreads, 4) drift_partials_kernel(const T* __
 }
 
 // Fixed-order reduction of the CTA partials; result = {rel, num, den}.
+// {rel, num, den} of the drift from its two sums (zero denominator: 0 when
+// the numerator is 0, else +inf).
+__device__ __forceinline__ void write_drift_result(double num, double den, double* result) {
+  double rel;
+  if (den == 0.0) rel = (num == 0.0) ? 0.0 : INFINITY;
+  else rel = num / den;
+  result[0] = rel;
+  result[1] = num;
+  result[2] = den;
+}
+
 __global__ void __launch_bounds__(kThreads) drift_final_kernel(const double2* __restrict__ partials, int nparts,
                                                                double* __restrict__ result) {
   double n = 0.0, d = 0.0;
@@ -156,15 +167,7 @@ __global__ void __launch_bounds__(kThreads) drift_final_kernel(const double2* __
     }
     __syncthreads();
   }
-  if (threadIdx.x == 0) {
-    const double num = sn[0], den = sd[0];
-    double rel;
-    if (den == 0.0) rel = (num == 0.0) ? 0.0 : INFINITY;
-    else rel = num / den;
-    result[0] = rel;
-    result[1] = num;
-    result[2] = den;
-  }
+  if (threadIdx.x == 0) write_drift_result(sn[0], sd[0], result);
 }
 
 template <typename T>
@@ -325,7 +328,8 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
                                                                             const float* __restrict__ scc,
                                                                             const float* __restrict__ shp,
                                                                             const float* __restrict__ scp, float eps,
-                                                                            double2* __restrict__ partials) {
+                                                                            double2* __restrict__ partials,
+                                                                            unsigned int* done, double* result) {
   extern __shared__ __align__(128) uint8_t tsm[];
   const int nwarps = blockDim.x >> 5;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -341,9 +345,11 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
   const int64_t gw = (int64_t)blockIdx.x * nwarps + warp, nw = (int64_t)gridDim.x * nwarps;
   const int64_t n_my = (step > 0 && gw < rows) ? (rows - 1 - gw) / nw + 1 : 0;
   const uint32_t row_bytes = (uint32_t)d * sizeof(float);
+  // rows from the last one down: the patch embedding that writes h_cur just
+  // before this kernel leaves its last rows in L2, so they are read first
   auto issue = [&](int64_t k) {
     const int st = (int)(k % kTemniStages);
-    const int64_t row = gw + k * nw;
+    const int64_t row = rows - 1 - (gw + k * nw);
     mbar_expect_tx(&wf[st], 2 * row_bytes);
     bulk_load(wr + (size_t)st * 2 * d, xc + row * d, row_bytes, &wf[st]);
     bulk_load(wr + (size_t)st * 2 * d + d, xp + row * d, row_bytes, &wf[st]);
@@ -460,6 +466,32 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
     }
     partials[blockIdx.x] = make_double2(dn, dd);
   }
+  // With a done counter (zero on entry), the CTA that finishes last sums the
+  // partials in a fixed order and writes the result, then sets the counter
+  // back to zero: no second launch.
+  if (done != nullptr) {
+    __shared__ bool last;
+    if (threadIdx.x == 0) {
+      __threadfence();  // this CTA's partial is visible before it is counted
+      last = atomicAdd(done, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (last && warp == 0) {
+      __threadfence();
+      double n = 0.0, e = 0.0;
+      for (int i = lane; i < (int)gridDim.x; i += 32) {
+        const double2 p = __ldcg(&partials[i]);
+        n += p.x;
+        e += p.y;
+      }
+      n = warp_sum_d(n);
+      e = warp_sum_d(e);
+      if (lane == 0) {
+        write_drift_result(n, e, result);
+        *done = 0u;
+      }
+    }
+  }
 }
 
 // ---------------------------------------------------------------- GEMV
@@ -540,6 +572,35 @@ __global__ void patchify_kernel(const float* __restrict__ lat, TO* __restrict__ 
     const int c = p;
     const int64_t src = (((int64_t)c * F + (f * pt + dt)) * H + (h * ph + dh)) * W + (w * pw + dw);
     io<TO>::st(tok + i, lat[src]);
+  }
+}
+
+// The same gather into bf16 tokens of width 2P that carry each fp32 value as
+// the sum of two bf16 parts: hi = bf16(x) in column p, lo = bf16(x - hi) in
+// column P + p.  x - hi is exact in fp32 and lo rounds it to 8 bits, so
+// hi + lo equals x to within 2^-17 |x|; a bf16 GEMM against the weights
+// repeated along K ([W | W]) then forms the fp32-input patch embedding on
+// tensor cores.
+__global__ void patchify_split_kernel(const float* __restrict__ lat, __nv_bfloat16* __restrict__ tok, int C, int F,
+                                      int H, int W, int pt, int ph, int pw) {
+  const int Hp = H / ph, Wp = W / pw;
+  const int P = C * pt * ph * pw;
+  const int64_t total = (int64_t)(F / pt) * Hp * Wp * P;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+    const int64_t n = i / P;
+    int p = (int)(i % P);
+    const int p0 = p;
+    const int f = (int)(n / ((int64_t)Hp * Wp)), h = (int)((n / Wp) % Hp), w = (int)(n % Wp);
+    const int dw = p % pw; p /= pw;
+    const int dh = p % ph; p /= ph;
+    const int dt = p % pt; p /= pt;
+    const int c = p;
+    const int64_t src = (((int64_t)c * F + (f * pt + dt)) * H + (h * ph + dh)) * W + (w * pw + dw);
+    const float x = lat[src];
+    const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+    tok[n * 2 * P + p0] = hi;
+    tok[n * 2 * P + P + p0] = __float2bfloat16_rn(x - __bfloat162float(hi));
   }
 }
 
@@ -713,7 +774,7 @@ acid_status ln_mod(int in_dtype, const void* x, int out_dtype, void* y, int64_t 
 template <int NV4, bool HOLD>
 acid_status launch_temni_drift(const float* h_cur, const float* h_prev, const float* mod_cur, const float* mod_prev,
                                const int* step_dev, int step_host, int64_t rows, int d, float eps, double2* parts,
-                               cudaStream_t s, int* grid_out) {
+                               unsigned int* done, double* result, cudaStream_t s, int* grid_out) {
   constexpr int kSmemMax = 226 * 1024;  // dynamic shared memory, below the 227 KB limit less the static part
   static bool attr_done = false;
   if (!attr_done) {
@@ -730,7 +791,8 @@ acid_status launch_temni_drift(const float* h_cur, const float* h_prev, const fl
   const int grid = (int)std::min<int64_t>(std::min<int64_t>(kDriftMaxBlocks, (int64_t)num_sms_elem()),
                                           std::max<int64_t>(1, (rows + warps - 1) / warps));
   temni_drift_kernel<NV4, HOLD><<<grid, 32 * warps, smem, s>>>(h_cur, h_prev, step_dev, step_host, rows, d, mod_cur,
-                                                               mod_cur + d, mod_prev, mod_prev + d, eps, parts);
+                                                               mod_cur + d, mod_prev, mod_prev + d, eps, parts,
+                                                               done, result);
   ACID_CHECK_LAUNCH();
   *grid_out = grid;
   return ACID_OK;
@@ -738,7 +800,7 @@ acid_status launch_temni_drift(const float* h_cur, const float* h_prev, const fl
 
 acid_status temni_drift(const float* h_cur, const float* h_prev, const float* mod_cur, const float* mod_prev,
                         const int* step_dev, int step_host, int64_t rows, int d, float eps, double* d_result,
-                        void* workspace, size_t ws_bytes, cudaStream_t s) {
+                        void* workspace, size_t ws_bytes, cudaStream_t s, unsigned int* done) {
   ACID_REQUIRE(d % 8 == 0 && d <= 3072, ACID_ERR_UNSUPPORTED, "temni_drift: d must be a multiple of 8, <= 3072");
   ACID_REQUIRE(ws_bytes >= sizeof(double2) * kDriftMaxBlocks, ACID_ERR_WORKSPACE, "temni_drift: workspace too small");
   ACID_REQUIRE(aligned(h_cur, 16) && aligned(h_prev, 16) && aligned(mod_cur, 16) && aligned(mod_prev, 16),
@@ -747,16 +809,18 @@ acid_status temni_drift(const float* h_cur, const float* h_prev, const float* mo
   ProfScope prof(PROF_DRIFT, (double)rows * d * 8.0, s);  // read both steps' H_in (fp32)
   int grid = 1;
   if (d <= 512)
-    ACID_TRY((launch_temni_drift<4, true>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts, s,
-                                         &grid)));
+    ACID_TRY((launch_temni_drift<4, true>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts, done,
+                                         d_result, s, &grid)));
   else if (d <= 1536)
     ACID_TRY((launch_temni_drift<12, true>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts,
-                                          s, &grid)));
+                                          done, d_result, s, &grid)));
   else
     ACID_TRY((launch_temni_drift<24, false>(h_cur, h_prev, mod_cur, mod_prev, step_dev, step_host, rows, d, eps, parts,
-                                           s, &grid)));
-  drift_final_kernel<<<1, kThreads, 0, s>>>(parts, grid, d_result);
-  ACID_CHECK_LAUNCH();
+                                           done, d_result, s, &grid)));
+  if (done == nullptr) {
+    drift_final_kernel<<<1, kThreads, 0, s>>>(parts, grid, d_result);
+    ACID_CHECK_LAUNCH();
+  }
   return ACID_OK;
 }
 
@@ -811,6 +875,14 @@ acid_status patchify(const float* latent, int out_dtype, void* tokens, int C, in
     patchify_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(latent, (__nv_bfloat16*)tokens, C, F, H, W, pt, ph, pw);
   else
     patchify_kernel<float><<<grid, kThreads, 0, s>>>(latent, (float*)tokens, C, F, H, W, pt, ph, pw);
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+acid_status patchify_split(const float* latent, void* tokens, int C, int F, int H, int W, int pt, int ph, int pw,
+                           cudaStream_t s) {
+  const int64_t total = (int64_t)C * F * H * W;
+  patchify_split_kernel<<<grid_for(total), kThreads, 0, s>>>(latent, (__nv_bfloat16*)tokens, C, F, H, W, pt, ph, pw);
   ACID_CHECK_LAUNCH();
   return ACID_OK;
 }

@@ -88,10 +88,12 @@ acid_status ln_mod(int in_dtype, const void* x, int out_dtype, void* y, int64_t 
 // and their block-0 modulations (shift then scale, d each): TEMNI of both
 // steps formed in registers, 8 bytes read per element.  Result {rel, num, den}
 // in d_result as drift_launch.  step from step_dev (device) if non-null, else
-// step_host; step 0 gives zero sums.
+// step_host; step 0 gives zero sums.  done: null, or a device counter that is
+// zero on entry; then the kernel's last CTA forms the result (one launch) and
+// leaves the counter at zero again.
 acid_status temni_drift(const float* h_cur, const float* h_prev, const float* mod_cur, const float* mod_prev,
                         const int* step_dev, int step_host, int64_t rows, int d, float eps, double* d_result,
-                        void* workspace, size_t ws_bytes, cudaStream_t s);
+                        void* workspace, size_t ws_bytes, cudaStream_t s, unsigned int* done = nullptr);
 
 // y[j] = sum_k W[j, k] act(x[k]) + b[j]; act = SiLU if silu_input.
 acid_status gemv(int w_dtype, const void* W, const float* b, const float* x, float* y, int n_out,
@@ -114,6 +116,10 @@ acid_status add_mixed(int a_dtype, const void* a, int b_dtype, const void* b, in
 
 acid_status patchify(const float* latent, int out_dtype, void* tokens, int C, int F, int H, int W,
                      int pt, int ph, int pw, cudaStream_t s);
+// bf16 tokens [N, 2P]: each fp32 patch value x as hi = bf16(x) in column p and
+// lo = bf16(x - hi) in column P + p (hi + lo = x to within 2^-17 |x|)
+acid_status patchify_split(const float* latent, void* tokens, int C, int F, int H, int W, int pt, int ph, int pw,
+                           cudaStream_t s);
 // v (optional) = unpatchify(vtok); latent += dsigma * v
 acid_status unpatchify_euler(const float* vtok, float* v_out, float* latent, int C, int F, int H,
                              int W, int pt, int ph, int pw, float dsigma, cudaStream_t s);

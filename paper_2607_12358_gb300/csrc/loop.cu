@@ -28,7 +28,7 @@ struct LoopWs {
   float* temb;
   float* mod0[2];   // block 0 shift / scale (TEMNI) of the even / odd steps
   float* fmod;      // final layer shift / scale
-  uint8_t* tokens;  // [N, P] fp32 patch vectors
+  uint8_t* tokens;  // [N, P] fp32 patch vectors, or [N, 2P] bf16 hi / lo parts (patch_split)
   float* h_in[2];   // [N, d] patch embedding (fp32) of the even / odd steps
   float* temni[2];  // [N, d] DiCache probe features of the even / odd steps
   float* resid;     // [N, d] TeaCache residual H_out - H_in
@@ -48,6 +48,11 @@ struct LoopWs {
   int* dc_count;    // computed steps cached (0, 1, 2)
   double* dres;     // [8] device drift results
   uint8_t* drift_ws;
+  unsigned int* drift_done;  // TEMNI drift: CTAs finished (zero between launches)
+  // bf16 models with P % 8 == 0: the patch embedding runs on tensor cores
+  // against the patch weights repeated along K, [d, 2P] bf16
+  bool patch_split;
+  uint8_t* patch_w2;
   float2* rope;
   uint8_t* block_base;
   // device-side loop state for graph-launched generations
@@ -136,6 +141,9 @@ LoopWs loop_layout(const acid_model& m, void* base) {
   w.dc_count = b.take<int>(1);
   w.dres = b.take<double>(8);
   w.drift_ws = b.take<uint8_t>(drift_workspace_bytes(0));
+  w.drift_done = b.take<unsigned int>(1);
+  w.patch_split = dt == ACID_BF16 && s.P % 8 == 0;
+  w.patch_w2 = b.take<uint8_t>(w.patch_split ? (size_t)s.d * 2 * s.P * 2 : 0);
   RopeTable rt = rope_layout(m.block.grid_f, m.block.grid_h, m.block.grid_w, m.block.d / std::max(1, m.block.heads));
   w.rope = b.take<float2>((size_t)rt.elems());
   // one block workspace, sized for the larger of the first and last block kinds
@@ -427,6 +435,13 @@ extern "C" acid_status acid_loop_begin(const acid_model* m, const acid_loop_cfg*
   RopeTable rt = rope_layout(m->block.grid_f, m->block.grid_h, m->block.grid_w, m->block.d / m->block.heads);
   ACID_TRY(rope_build(rt, w.rope, m->block.rope_theta, s));
   ACID_CUDA(cudaMemsetAsync(w.dc_count, 0, sizeof(int), s));
+  ACID_CUDA(cudaMemsetAsync(w.drift_done, 0, sizeof(unsigned int), s));
+  if (w.patch_split) {  // [W | W]: each row of the patch weights twice
+    const size_t row = (size_t)sh.P * 2;
+    for (int k = 0; k < 2; ++k)
+      ACID_CUDA(cudaMemcpy2DAsync(w.patch_w2 + k * row, 2 * row, m->patch.w, row, row, sh.d, cudaMemcpyDeviceToDevice,
+                                  s));
+  }
   ACID_REQUIRE(cfg->method != ACID_METHOD_DICACHE || cfg->probe_blocks <= total_blocks(*m), ACID_ERR_INVALID_ARG,
                "acid_loop_begin: probe_blocks exceeds the number of blocks");
   return ACID_OK;
@@ -467,6 +482,24 @@ struct StepTimer {
 // unchanged and points *v_out at the branch's velocity (fp32, latent layout,
 // inside w).  Fills the step log's fields except ms; does not advance
 // st->step.
+// Patch embedding H_in (fp32) of the latent.  bf16 models: the tokens as
+// bf16 hi + lo parts against the weights repeated along K, one tcgen05 GEMM
+// with fp32 accumulation (the fp32 tokens to within 2^-17 relative); fp32
+// models: the fp32 SIMT GEMM.
+static acid_status patch_embed(const acid_model& m, const LoopWs& w, const float* latent, float* h_in,
+                               cudaStream_t s) {
+  const Shape sh = shape_of(m);
+  Epilogue e;
+  e.bias = m.patch.b;
+  e.out_fp32 = true;
+  if (w.patch_split) {
+    ACID_TRY(patchify_split(latent, w.tokens, m.latent_c, m.latent_f, m.latent_h, m.latent_w, m.pt, m.ph, m.pw, s));
+    return linear_forward(ACID_BF16, w.tokens, 2 * sh.P, sh.N, (int)(2 * sh.P), w.patch_w2, sh.d, h_in, sh.d, e, s);
+  }
+  ACID_TRY(patchify(latent, ACID_FP32, w.tokens, m.latent_c, m.latent_f, m.latent_h, m.latent_w, m.pt, m.ph, m.pw, s));
+  return linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, m.block.dtype, m.patch.w, sh.d, h_in, sh.d, e, s);
+}
+
 static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, acid_loop_state* st, float* latent,
                                const LoopWs& w, bool defer_euler, const float** v_out, acid_step_log& lg,
                                cudaStream_t s) {
@@ -495,14 +528,7 @@ static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, ac
   // patch embedding H_in (fp32)
   // (fp32 tokens and accumulation: the drift signal compares consecutive H_in
   // that differ by a few percent, so it must not see bf16 input rounding)
-  ACID_TRY(patchify(latent, ACID_FP32, w.tokens, m->latent_c, m->latent_f, m->latent_h, m->latent_w, m->pt, m->ph,
-                    m->pw, s));
-  {
-    Epilogue e;
-    e.bias = m->patch.b;
-    e.out_fp32 = true;
-    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m->patch.w, sh.d, h_in, sh.d, e, s));
-  }
+  ACID_TRY(patch_embed(*m, w, latent, h_in, s));
   const int64_t vrow0 = m->block.kind == ACID_BLOCK_WAN ? 0 : sh.L;
   void* x_video = w.xbuf + vrow0 * sh.d * es(dt);
   auto run_model = [&]() -> acid_status {
@@ -518,7 +544,7 @@ static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, ac
     // block-0 modulation in one read-only pass
     ACID_TRY(gemv(dt, m->blocks[0].mod.w, m->blocks[0].mod.b, w.temb, w.mod0[par], 2 * sh.d, sh.d, true, s));
     ACID_TRY(temni_drift(h_in, w.h_in[par ^ 1], w.mod0[par], w.mod0[par ^ 1], nullptr, i, sh.N, sh.d,
-                         m->block.ln_eps, w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+                         m->block.ln_eps, w.dres, w.drift_ws, drift_workspace_bytes(0), s, w.drift_done));
     if (!warm) {
       ACID_REQUIRE(i > 0, ACID_ERR_INVALID_ARG, "TeaCache needs at least one warmup step");
       double h[3];
@@ -854,13 +880,7 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
   ACID_TRY(timestep_sinusoid_sig(w.sinus, w.sig, step, m.time_freq_dim, s));
   ACID_TRY(gemv(dt, m.time1.w, m.time1.b, w.sinus, w.temb_h, sh.d, m.time_freq_dim, false, s));
   ACID_TRY(gemv(dt, m.time2.w, m.time2.b, w.temb_h, w.temb, sh.d, sh.d, true, s));
-  ACID_TRY(patchify(latent, ACID_FP32, w.tokens, m.latent_c, m.latent_f, m.latent_h, m.latent_w, m.pt, m.ph, m.pw, s));
-  {
-    Epilogue e;
-    e.bias = m.patch.b;
-    e.out_fp32 = true;
-    ACID_TRY(linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, dt, m.patch.w, sh.d, h_in, sh.d, e, s));
-  }
+  ACID_TRY(patch_embed(m, w, latent, h_in, s));
   // ---- signal and decision
   float* v = w.v[0];
   float* v_prev = w.v[1];
@@ -871,7 +891,7 @@ acid_status capture_branch(const acid_model& m, const acid_loop_cfg& cfg, LoopWs
   if (cfg.method == ACID_METHOD_TEACACHE) {
     ACID_TRY(gemv(dt, m.blocks[0].mod.w, m.blocks[0].mod.b, w.temb, w.mod0[par], 2 * sh.d, sh.d, true, s));
     ACID_TRY(temni_drift(h_in, w.h_in[par ^ 1], w.mod0[par], w.mod0[par ^ 1], step, 0, sh.N, sh.d, m.block.ln_eps,
-                         w.dres, w.drift_ws, drift_workspace_bytes(0), s));
+                         w.dres, w.drift_ws, drift_workspace_bytes(0), s, w.drift_done));
   } else if (cfg.method == ACID_METHOD_DICACHE) {
     if (vrow0 > 0) ACID_CUDA(cudaMemcpyAsync(w.xbuf, w.text, sh.L * sh.d * es(dt), cudaMemcpyDeviceToDevice, s));
     ACID_TRY(add_mixed(ACID_FP32, h_in, ACID_FP32, h_in, dt, x_video, sh.N * sh.d, 0.0f, s));

@@ -248,3 +248,34 @@ def test_teacache_signal_across_row_widths(acid, d):
     for i in range(cfg.warmup, cfg.steps):
         ref = O.rel_l1(temni[i - 1], temni[i])
         assert abs(logs[i]["signal"] - ref) <= 1e-3 * ref, (d, i, logs[i]["signal"], ref)
+
+
+def test_bf16_patch_embedding_keeps_fp32_tokens(acid):
+    """bf16 models form the patch embedding H_in on tensor cores from the fp32
+    tokens split into bf16 hi and lo parts (hi + lo = x to within 2^-17 |x|).
+    The first steps of a 1000-step schedule change the latent by about 0.1%
+    per step, so the TeaCache signal is near 2e-3; rounding the tokens to bf16
+    alone would move it by about 3% there, the hi + lo split by about 2e-7
+    (both computed with the oracle).  The signal must match the oracle's
+    (fp32 tokens, fp64 arithmetic) to 1e-4 relative."""
+    cfg = S.get_config("wan", d=256, heads=2, ffn=512, n_blocks=1, n_text=40, d_text=256, latent_f=5,
+                       latent_h=32, latent_w=46, steps=1000)
+    w = S.model_weights(cfg, 8)
+    lat = S.latent(cfg, 8)
+    text = S.text(cfg, 8)
+    model = acid.DeviceModel(cfg, w, DEV)
+    c, keep = acid.loop_cfg(cfg)
+    loop = acid.Loop(model, c, torch.from_numpy(text).to(DEV, torch.bfloat16), DEV)
+    tl = torch.from_numpy(lat).to(DEV)
+    xs, logs = [], []
+    for i in range(4):
+        xs.append(tl.cpu().numpy().astype(np.float64))
+        logs.append(acid.log_to_dict(loop.step(tl)))
+    acid.check_device_error()
+    sig = O.sigmas(cfg.steps)
+    temni = [O.block0_temni(cfg, w, O.step_inputs(cfg, w, x, 1000 * sig[i], with_blocks=False).h_in,
+                            O.time_embedding(1000 * sig[i], w, cfg.time_freq_dim)) for i, x in enumerate(xs)]
+    for i in range(cfg.warmup, len(xs)):
+        ref = O.rel_l1(temni[i - 1], temni[i])
+        assert ref < 1e-2, ref
+        assert abs(logs[i]["signal"] - ref) <= 1e-4 * ref, (i, logs[i]["signal"], ref)
