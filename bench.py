@@ -528,7 +528,7 @@ def run_ours(args) -> None:
         "attention_tflops": att_tflops,
         "attention_pct_bf16_peak": 100.0 * att_tflops / peaks["bf16_tflops"],
         "linear": {"tflops": lin_tflops, "launches": l_n, "ms": l_ms},
-        "drift": {"kernel": "temni_drift_kernel (TEMNI of this and the previous step formed from both steps' fp32 H_in in one read-only pass, 8 B/elem) + drift_final_kernel",
+        "drift": {"kernel": "temni_drift_kernel (TEMNI of this and the previous step formed from both steps' fp32 H_in in one read-only pass, 8 B/elem; its last CTA reduces the partials)",
                   "gbs": d_gbs, "frac_of_hbm": d_gbs / peaks["hbm_gbs"] if d_gbs else None,
                   "hbm_peak_source": f"hbm_gbs, {src}", "launches": d_n, "ms": d_ms},
         "block_ms": t_max / K / cfg.n_blocks,

@@ -195,6 +195,27 @@ __global__ void add_mixed_kernel(const TA* __restrict__ a, const TB* __restrict_
     io<TO>::st(out + i, io<TA>::ld(a + i) + bs * io<TB>::ld(b + i));
 }
 
+// The same on eight consecutive values per thread (16-byte aligned operands);
+// READ_B false: out = a (b_scale 0, b not read).
+template <typename TA, typename TB, typename TO, bool READ_B>
+__global__ void add_mixed8_kernel(const TA* __restrict__ a, const TB* __restrict__ b, TO* out, int64_t n, float bs) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (int64_t i = tid; i < n / 8; i += stride) {
+    float x[8];
+    load8(a + 8 * i, x);
+    if constexpr (READ_B) {
+      float y[8];
+      load8(b + 8 * i, y);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) x[j] = x[j] + bs * y[j];
+    }
+    store8(out + 8 * i, x);
+  }
+  for (int64_t i = n / 8 * 8 + tid; i < n; i += stride)
+    io<TO>::st(out + i, READ_B ? io<TA>::ld(a + i) + bs * io<TB>::ld(b + i) : io<TA>::ld(a + i));
+}
+
 // ---------------------------------------------------------------- LayerNorm
 // One warp per row; row kept in registers (d <= 256 * kMaxV).
 constexpr int kLnMaxV = 12;
@@ -319,6 +340,21 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
                : "memory");
 }
 
+// The same with an L2 cache policy for the source lines.
+__device__ __forceinline__ void bulk_load_hint(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
+                                               uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
 template <int NV4, bool HOLD>
 __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(const float* __restrict__ xc,
                                                                             const float* __restrict__ xp,
@@ -345,14 +381,18 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
   const int64_t gw = (int64_t)blockIdx.x * nwarps + warp, nw = (int64_t)gridDim.x * nwarps;
   const int64_t n_my = (step > 0 && gw < rows) ? (rows - 1 - gw) / nw + 1 : 0;
   const uint32_t row_bytes = (uint32_t)d * sizeof(float);
-  // rows from the last one down: the patch embedding that writes h_cur just
-  // before this kernel leaves its last rows in L2, so they are read first
+  // Rows from the last one down: the patch embedding that writes h_cur just
+  // before this kernel leaves its last rows in L2 (dirty), so they are read
+  // first.  The previous step's rows are not read again in this step: they
+  // are loaded evict-first, so that they, and not those dirty h_cur lines,
+  // give way to new lines, and no write-back of h_cur falls into this kernel.
+  const uint64_t prev_policy = l2_policy_evict_first();
   auto issue = [&](int64_t k) {
     const int st = (int)(k % kTemniStages);
     const int64_t row = rows - 1 - (gw + k * nw);
     mbar_expect_tx(&wf[st], 2 * row_bytes);
     bulk_load(wr + (size_t)st * 2 * d, xc + row * d, row_bytes, &wf[st]);
-    bulk_load(wr + (size_t)st * 2 * d + d, xp + row * d, row_bytes, &wf[st]);
+    bulk_load_hint(wr + (size_t)st * 2 * d + d, xp + row * d, row_bytes, &wf[st], prev_policy);
   };
   // each warp's first copies are issued before the modulation vectors are
   // staged, so their latency overlaps the staging
@@ -719,10 +759,15 @@ acid_status add_same(int dtype, const void* a, const void* b, void* out, int64_t
 
 acid_status add_mixed(int ad, const void* a, int bd, const void* b, int od, void* out, int64_t n, float bs,
                       cudaStream_t s) {
-  const int grid = grid_for(n);
   using H = __nv_bfloat16;
-#define ACID_ADD(TA, TB, TO) \
-  add_mixed_kernel<TA, TB, TO><<<grid, kThreads, 0, s>>>((const TA*)a, (const TB*)b, (TO*)out, n, bs)
+  const bool vec = aligned(a, 16) && aligned(b, 16) && aligned(out, 16);
+  const int grid = vec ? grid_for(n / 8 + 1, kThreads, 152 * 8) : grid_for(n);
+#define ACID_ADD(TA, TB, TO)                                                                                   \
+  (!vec ? add_mixed_kernel<TA, TB, TO><<<grid, kThreads, 0, s>>>((const TA*)a, (const TB*)b, (TO*)out, n, bs)  \
+   : bs == 0.0f                                                                                                \
+       ? add_mixed8_kernel<TA, TB, TO, false><<<grid, kThreads, 0, s>>>((const TA*)a, (const TB*)b, (TO*)out, n, \
+                                                                       bs)                                   \
+       : add_mixed8_kernel<TA, TB, TO, true><<<grid, kThreads, 0, s>>>((const TA*)a, (const TB*)b, (TO*)out, n, bs))
   const int key = ad * 4 + bd * 2 + od;  // ACID_BF16 = 0, ACID_FP32 = 1
   switch (key) {
     case 0: ACID_ADD(H, H, H); break;

@@ -380,6 +380,117 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
   }
 }
 
+// Bias of a chunk's 32 columns, the same for every lane (broadcast loads
+// through the read-only path; 16-byte loads where the vector is aligned).
+__device__ __forceinline__ void load_bias32(const EpiDev& e, int col0, float* bias) {
+  if (e.bias == nullptr) {
+#pragma unroll
+    for (int k = 0; k < 32; ++k) bias[k] = 0.f;
+  } else if ((reinterpret_cast<uintptr_t>(e.bias + col0) & 15) == 0) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float4 t = __ldg(reinterpret_cast<const float4*>(e.bias + col0) + k);
+      bias[4 * k] = t.x; bias[4 * k + 1] = t.y; bias[4 * k + 2] = t.z; bias[4 * k + 3] = t.w;
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 32; ++k) bias[k] = __ldg(e.bias + col0 + k);
+  }
+}
+
+// Epilogue of one 32-row x 32-column chunk of a kind without a residual, in
+// the layout tcgen05.ld delivers (thread = row, 32 consecutive columns): the
+// bias and the kind's arithmetic in registers, then the output box written
+// once into the warp's stage in the tensor store's swizzled layout (fp32:
+// 128-byte rows, 16-byte unit u of row r at u ^ (r & 7); bf16: 64-byte rows,
+// unit u at u ^ ((r >> 1) & 3); both place the 32 rows' units of a given u in
+// distinct bank groups) and handed to one TMA store, which clips rows past M.
+// Shared-memory traffic is one write and one TMA read of the box.  The caller
+// makes sure the store that last read this stage has finished reading.
+template <int KIND, bool O32>
+__device__ __forceinline__ void epilogue_rows(const GemmDims& g, const EpiDev& e, const CUtensorMap* tmO,
+                                              uint8_t* stage, int64_t row0, int col0, const uint32_t* r,
+                                              const float* bias) {
+  const int lane = threadIdx.x & 31;
+  uint64_t v[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k)
+    v[k] = f2_add(f2_pack(__uint_as_float(r[2 * k]), __uint_as_float(r[2 * k + 1])),
+                  f2_pack(bias[2 * k], bias[2 * k + 1]));
+  if constexpr (KIND == EPI_GELU) {
+#pragma unroll
+    for (int k = 0; k < 16; ++k) v[k] = gelu_x2(v[k]);
+  } else if constexpr (KIND == EPI_ROPE_QKV) {
+    // the chunk's 16 pairs lie in one head (head_dim is a power of two >= 32)
+    const int64_t row = row0 + lane, grow = row + e.row_base;
+    if (col0 < 2 * e.d && grow >= e.rope_first_video && row < g.M) {
+      const RopePos pp = rope_pos(e.rope, (int)(grow - e.rope_first_video));
+      const int j0 = (col0 & (e.head_dim - 1)) >> 1;
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const float2 cs = __ldg(&rope_cs_ptr(e.rope, pp, j0 + k));
+        float x0, x1;
+        f2_unpack(v[k], x0, x1);
+        v[k] = f2_pack(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
+      }
+    }
+  }
+  if constexpr (O32) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      float a0, a1, a2, a3;
+      f2_unpack(v[2 * u], a0, a1);
+      f2_unpack(v[2 * u + 1], a2, a3);
+      *reinterpret_cast<float4*>(stage + lane * 128 + ((u ^ (lane & 7)) << 4)) = make_float4(a0, a1, a2, a3);
+    }
+  } else {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      uint32_t w[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float a0, a1;
+        f2_unpack(v[4 * u + q], a0, a1);
+        w[q] = pack_bf16(a0, a1);
+      }
+      *reinterpret_cast<uint4*>(stage + lane * 64 + ((u ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    tma_store_2d(tmO, stage, col0, (int)row0);
+    bulk_commit_group();
+  }
+}
+
+// One chunk of a kind without a residual: accumulator and bias loads, the
+// stage (bf16 output: two 2 KB stages per warp used in turn, so a chunk waits
+// only for the store before last; fp32 output: one 4 KB stage), epilogue_rows.
+template <int KIND, bool O32>
+__device__ __forceinline__ void tma_kind_chunk(const GemmDims& g, const EpiDev& e, const CUtensorMap* tmO,
+                                               uint8_t* stage, uint32_t taddr, int64_t row0, int col0, bool ok,
+                                               int& nstore) {
+  const int lane = threadIdx.x & 31;
+  uint32_t r[32];
+  float bias[32];
+  tmem_ld32(taddr, r);
+  const bool live = ok && row0 < g.M && col0 < g.N;
+  if (live) load_bias32(e, col0, bias);
+  tmem_wait_ld();
+  if (!live) return;
+  uint8_t* st = stage;
+  if constexpr (O32) {
+    if (lane == 0) bulk_wait_group_read<0>();
+  } else {
+    st += (nstore & 1) * 2048;
+    if (lane == 0) bulk_wait_group_read<1>();
+  }
+  __syncwarp();
+  epilogue_rows<KIND, O32>(g, e, tmO, st, row0, col0, r, bias);
+  ++nstore;
+}
+
 template <int BN, int KIND, bool R32, bool O32>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -675,13 +786,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     float* stage = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES) + (warp - 2) * C::EPI_STAGE_FLOATS;
     const uint32_t acc_empty0 = mapa_shared(smem_u32(acc_empty), 0);
-    int local = 0;
+    int local = 0, nstore = 0;
     for (int tile = pair; tile < num_tiles; tile += npairs, ++local) {
       const int b = local & 1, use = local >> 1;
       const int m_tile = tile / num_n, n_tile = tile % num_n;
       const bool ok = mbar_wait(&acc_full[b], use & 1);
       tc_fence_after();
       const int64_t row0 = (int64_t)m_tile * 2 * BM + (int64_t)rank * BM + q * 32;
+      if constexpr (kTmaStore<KIND>) {
+        constexpr int NC = BN / 64;
+        const int cbeg = half * (BN / 2);
+#pragma unroll 1
+        for (int i = 0; i < NC; ++i)
+          tma_kind_chunk<KIND, O32>(g, e, &tmO, reinterpret_cast<uint8_t*>(stage),
+                                    tmem + lane_base + b * BN + cbeg + 32 * i, row0, n_tile * BN + cbeg + 32 * i, ok,
+                                    nstore);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(acc_empty0 + 8 * b);
+        if (!ok) break;
+        continue;
+      }
       constexpr int NC = BN / 64;
       const int cbeg = half * (BN / 2);
       const int lcol = 4 * (lane & 7);
@@ -843,6 +968,10 @@ template <int KIND, bool R32, bool O32>
 int max_pairs() {
   static int n = -1;
   if (n < 0) {
+    // the dynamic shared memory limit must be raised before the query
+    if (cudaFuncSetAttribute(gemm_tc2_kernel<KIND, R32, O32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Tc2Cfg::SMEM) != cudaSuccess)
+      return 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * 76, 1, 1);
     cfg.blockDim = dim3(kGemmThreads, 1, 1);

@@ -152,6 +152,35 @@ def test_linear_bf16_pair_tiles(acid, M, K, N, epi, fp32):
     assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
 
 
+@pytest.mark.parametrize("K,epi,fp32", [(1536, "gated_res", True), (1536, "res", True), (1536, "bias", False),
+                                        (1536, "gelu", True), (8960, "gated_res", False)])
+def test_linear_bf16_wan_shapes_last_rows(acid, K, epi, fp32):
+    """The Wan-1.3B projections with N = 1536 over 32760 rows (output
+    projections, cross-attention query, FFN2) and a GELU output, at full size:
+    the persistent launch's last, partly filled round of tiles and the ragged
+    last row tile (32760 = 255 x 128 + 120).  Every one of the last 640 rows,
+    and rows spread over the rest, are compared with the oracle."""
+    M, N = 32760, 1536
+    rng = np.random.default_rng(K + N)
+    a = S.round_to_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    w = S.round_to_bf16((0.03 * rng.normal(size=(N, K))).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32)
+    g = rng.normal(size=N).astype(np.float32)
+    r = rng.normal(size=(M, N)).astype(np.float32)
+    if not fp32:
+        r = S.round_to_bf16(r)
+    # the residual has the output's dtype and is updated in place
+    out = _f32(r) if fp32 else _bf(r)
+    acid.acid_linear_forward(_bf(a), _bf(w), _f32(b), epilogue=epi, gate=_f32(g),
+                             residual=out if epi in ("gated_res", "res") else None, out=out, out_fp32=fp32)
+    rows = np.array(sorted(set(range(M - 640, M)) | set(rng.integers(0, M - 640, size=64).tolist()) | {0, 1}))
+    acc = O.linear(a[rows], w, b)
+    ref = {"bias": acc, "gelu": O.gelu_tanh(acc), "gated_res": r[rows] + g * acc, "res": r[rows] + acc}[epi]
+    got = out[torch.from_numpy(rows).to(DEV)].float().cpu().numpy()
+    tol = 1e-4 if (fp32 and epi != "gelu") else 2 ** -8
+    assert np.abs(got - ref).max() <= tol * (np.abs(ref).max() + 1), np.abs(got - ref).max()
+
+
 def test_linear_bf16_offsets_past_32_bits(acid):
     """An output of 262181 x 8960 fp32 values (2.35e9 elements, 9.4 GB),
     updated in place by the gated-residual epilogue.  Rows from 239675 on
