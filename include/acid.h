@@ -385,7 +385,11 @@ acid_status acid_loop_workspace_size(const acid_model* m, size_t* bytes);
 /* Prepares a generation: zeroes `state`, projects the text features (WAN) or
  * stores the text tokens (COG/HV) into the workspace.  WAN with text also
  * computes every block's cross-attention keys and values from the projected
- * text there, once; the steps read them (acid_cond.ctx_kv).
+ * text there, once; the steps read them (acid_cond.ctx_kv).  bf16 models also
+ * get the patch weights repeated along K ([W | W]) for the tensor-core patch
+ * embedding, and the TEMNI drift's CTA counter is zeroed.  The whole
+ * workspace is the generation's state: to resume a generation elsewhere, copy
+ * all of it (with `state`).
  *   text      device [n_text, d_text] in the model dtype, or NULL if n_text = 0.
  *   workspace device, >= acid_loop_workspace_size bytes, 1024-byte aligned;
  *             holds the caches between steps, so the same workspace must be
