@@ -317,8 +317,9 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
 // scale).  Both TEMNI rows are formed in registers from the fp32 patch
 // embeddings H_in_t (xc) and H_in_{t-1} (xp), so the kernel reads 8 bytes per
 // element and writes nothing but one fp64 partial pair per CTA (reduced by
-// drift_final_kernel).
-// One warp per row pair (rows gw, gw + total warps, ...), reductions by warp
+// drift_final_kernel, or with a done counter by the CTA that finishes last).
+// One warp per row pair (rows counted from the end: gw, gw + total warps, ...
+// from the last row down), reductions by warp
 // shuffles only.  Lane 0 of each warp streams the warp's row pairs into its
 // own two-stage shared-memory ring with 1D bulk copies (completion counted on
 // the stage's mbarrier), so the bytes in flight come from shared memory, not
