@@ -82,6 +82,25 @@ acid_status acid_check_device_error(void);
  * stays usable.  Synchronises `stream`. */
 acid_status acid_selftest_wait_timeout(int64_t budget_cycles, acid_stream_t stream);
 
+/* Memory-index checks of the debug build.  The library built with
+ * `python -m paper_2607_12358_gb300.build --debug` (libacid_gb300_debug.so,
+ * compiled with ACID_BOUNDS_CHECK) checks the global-memory index of every
+ * hand-computed access in the element-wise, LayerNorm, drift, patch, GEMV,
+ * GEMM-epilogue and attention-merge kernels against the extent the host
+ * passed; an index outside it is not accessed and the first one per source
+ * file is recorded.  Accesses by the TMA engine are bounded by their tensor
+ * maps.  Synchronises the device and reports, then clears, the first
+ * recorded violation: *site = 0 if there is none, else a kernel-site code,
+ * with the index and the extent.  *checked = 1 in the debug build, 0 in the
+ * release build (which records nothing). */
+acid_status acid_bounds_report(int32_t* checked, int64_t* site, int64_t* index, int64_t* extent);
+
+/* Diagnostic of the index checks: one thread evaluates a check one past the
+ * end of an extent of 1000, with no memory access behind it.  In the debug
+ * build the next acid_bounds_report gives site 99, index 1000, extent 1000.
+ * Synchronises `stream`. */
+acid_status acid_selftest_bounds(acid_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Tracing: launch counting and per-launch device timing                     */
 /* ------------------------------------------------------------------------ */

@@ -9,7 +9,10 @@ from __future__ import annotations
 import ctypes as C
 import os
 
-_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libacid_gb300.so")
+# ACID_LIBRARY=debug selects the debug build (kernel memory-index checks, see
+# acid_bounds_report in include/acid.h), built by `build.py --debug`.
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                         "libacid_gb300_debug.so" if os.environ.get("ACID_LIBRARY") == "debug" else "libacid_gb300.so")
 
 ACID_OK, ACID_ERR_INVALID_ARG, ACID_ERR_UNSUPPORTED, ACID_ERR_WORKSPACE, ACID_ERR_CUDA, ACID_ERR_TIMEOUT = range(6)
 ACID_BF16, ACID_FP32 = 0, 1
@@ -77,6 +80,9 @@ _PROTOS = {
     "acid_version": (C.c_char_p, []),
     "acid_check_device_error": (C.c_int, []),
     "acid_selftest_wait_timeout": (C.c_int, [C.c_int64, _P]),
+    "acid_bounds_report": (C.c_int, [C.POINTER(C.c_int32), C.POINTER(C.c_int64), C.POINTER(C.c_int64),
+                                     C.POINTER(C.c_int64)]),
+    "acid_selftest_bounds": (C.c_int, [_P]),
     "acid_launch_count": (C.c_int64, []),
     "acid_profile_enable": (C.c_int, [C.c_int32]),
     "acid_profile_read": (C.c_int, [C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double),

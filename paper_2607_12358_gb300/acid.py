@@ -61,6 +61,20 @@ def selftest_wait_timeout(budget_cycles: int, stream=None) -> None:
     check(load().acid_selftest_wait_timeout(int(budget_cycles), _stream(stream)))
 
 
+def bounds_report() -> dict:
+    """The first kernel memory-index violation recorded since the last report
+    (debug build only; ``checked`` is False in the release build)."""
+    c, site, idx, ext = C.c_int32(), C.c_int64(), C.c_int64(), C.c_int64()
+    check(load().acid_bounds_report(C.byref(c), C.byref(site), C.byref(idx), C.byref(ext)))
+    return {"checked": bool(c.value), "site": site.value, "index": idx.value, "extent": ext.value}
+
+
+def selftest_bounds(stream=None) -> None:
+    """Evaluates one index check one past the end (no access behind it); the
+    debug build's next bounds_report() shows site 99."""
+    check(load().acid_selftest_bounds(_stream(stream)))
+
+
 def launch_count() -> int:
     return int(load().acid_launch_count())
 

@@ -665,6 +665,7 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(AttnDev a, int item0, i
     for (int i = 0; i < D / 32; ++i) acc[i] = fmaf(w, a.part_o[slot * D + i * 32 + lane], acc[i]);
   }
   const float inv = 1.0f / L;
+  if (!ACID_IN_BOUNDS(kSiteAttnMerge, row * a.ldo + a.o_col + h * D + D - 1, a.nq * a.ldo)) return;
   __nv_bfloat16* op = static_cast<__nv_bfloat16*>(a.out) + row * a.ldo + a.o_col + h * D;
 #pragma unroll
   for (int i = 0; i < D / 32; ++i) op[i * 32 + lane] = __float2bfloat16_rn(acc[i] * inv);
@@ -789,6 +790,7 @@ __global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__
       if (i < per) o[i] = fmaf(p, vr[i * 32 + lane], o[i] * corr);
     m = mn;
   }
+  if (!ACID_IN_BOUNDS(kSiteAttnF32, row * ldo + o_col + h * D + D - 1, nq * ldo)) return;
 #pragma unroll
   for (int i = 0; i < kMaxPer; ++i)
     if (i < per) out[row * ldo + o_col + h * D + i * 32 + lane] = o[i] / l;
@@ -819,5 +821,6 @@ acid_status attention_forward(int dtype, const AttnArgs& x, cudaStream_t s) {
 }
 
 ACID_DEVICE_FLAG_READER(take_device_error_attention)
+ACID_BOUNDS_READER(take_bounds_attention)
 
 }  // namespace acid

@@ -14,6 +14,9 @@ namespace acid {
 
 unsigned int take_device_error_gemm();
 unsigned int take_device_error_attention();
+BoundsRecord take_bounds_elementwise();
+BoundsRecord take_bounds_gemm();
+BoundsRecord take_bounds_attention();
 
 namespace {
 thread_local std::string t_last_error;
@@ -136,9 +139,44 @@ __global__ void wait_selftest_kernel(long long limit) {
   __syncthreads();
   if (threadIdx.x == 0) (void)mbar_wait_limit(&bar, 0, limit);
 }
+
+// Evaluates one index check one past the end of an extent of n, with no
+// memory access behind it: a debug build records {kSiteSelftest, n, n}.
+__global__ void bounds_selftest_kernel(long long n, int* sink) {
+  if (threadIdx.x == 0 && !ACID_IN_BOUNDS(kSiteSelftest, n, n) && sink != nullptr) *sink = 1;
+}
 }  // namespace
 ACID_DEVICE_FLAG_READER(take_device_error_capi)
+ACID_BOUNDS_READER(take_bounds_capi)
 }  // namespace acid
+
+extern "C" acid_status acid_bounds_report(int32_t* checked, int64_t* site, int64_t* index, int64_t* extent) {
+  clear_error();
+  ACID_REQUIRE(checked && site && index && extent, ACID_ERR_INVALID_ARG, "acid_bounds_report: null argument");
+  ACID_CUDA(cudaDeviceSynchronize());
+  const BoundsRecord recs[4] = {take_bounds_elementwise(), take_bounds_gemm(), take_bounds_attention(),
+                                take_bounds_capi()};
+  *checked = kBoundsChecked ? 1 : 0;
+  *site = *index = *extent = 0;
+  for (const BoundsRecord& r : recs) {
+    ACID_REQUIRE(r.site >= 0, ACID_ERR_CUDA, "acid_bounds_report: record not readable");
+    if (r.site != 0 && *site == 0) {
+      *site = r.site;
+      *index = r.index;
+      *extent = r.extent;
+    }
+  }
+  return ACID_OK;
+}
+
+extern "C" acid_status acid_selftest_bounds(acid_stream_t stream) {
+  clear_error();
+  cudaStream_t s = (cudaStream_t)stream;
+  bounds_selftest_kernel<<<1, 32, 0, s>>>(1000, nullptr);
+  ACID_CHECK_LAUNCH();
+  ACID_CUDA(cudaStreamSynchronize(s));
+  return ACID_OK;
+}
 
 extern "C" acid_status acid_selftest_wait_timeout(int64_t budget_cycles, acid_stream_t stream) {
   clear_error();

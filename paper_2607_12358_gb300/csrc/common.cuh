@@ -79,6 +79,47 @@ static __device__ unsigned int g_device_error = 0;
     return v;                                                                      \
   }
 
+// Debug builds (compiled with ACID_BOUNDS_CHECK, libacid_gb300_debug.so)
+// check the global-memory index of the kernels' hand-computed accesses
+// against the extent the host passed: ACID_IN_BOUNDS(site, i, n) is true for
+// 0 <= i < n; otherwise it records the translation unit's first violation
+// {site, index, extent} and returns false, and the caller skips the access.
+// Release builds compile every check to `true`.  Accesses made by the TMA
+// engine are bounded by their tensor maps and are not checked here.
+enum BoundsSite : int {
+  kSiteDrift = 1, kSiteAdd = 2, kSiteLayerNorm = 3, kSiteTemni = 4, kSitePatchify = 5, kSiteUnpatchify = 6,
+  kSiteGemv = 7, kSiteGemmResidual = 8, kSiteGemmStore = 9, kSiteGemmRope = 10, kSiteGemmF32 = 11,
+  kSiteAttnMerge = 12, kSiteAttnF32 = 13, kSiteSelftest = 99
+};
+struct BoundsRecord {
+  long long site, index, extent;
+};
+static __device__ BoundsRecord g_bounds = {0, 0, 0};
+#ifdef ACID_BOUNDS_CHECK
+static __device__ __noinline__ bool bounds_fail(int site, long long i, long long n) {
+  if (atomicCAS(reinterpret_cast<unsigned long long*>(&g_bounds.site), 0ull, (unsigned long long)site) == 0ull) {
+    g_bounds.index = i;
+    g_bounds.extent = n;
+  }
+  return false;
+}
+#define ACID_IN_BOUNDS(site, i, n)                                                   \
+  (((long long)(i) >= 0 && (long long)(i) < (long long)(n)) ? true                   \
+                                                           : ::acid::bounds_fail((site), (long long)(i), (long long)(n)))
+constexpr bool kBoundsChecked = true;
+#else
+#define ACID_IN_BOUNDS(site, i, n) true
+constexpr bool kBoundsChecked = false;
+#endif
+// Host reader of the translation unit's record (cleared after reading).
+#define ACID_BOUNDS_READER(fname)                                                    \
+  BoundsRecord fname() {                                                             \
+    BoundsRecord r{0, 0, 0}, z{0, 0, 0};                                             \
+    if (cudaMemcpyFromSymbol(&r, g_bounds, sizeof(r)) != cudaSuccess) r.site = -1;   \
+    else if (r.site) cudaMemcpyToSymbol(g_bounds, &z, sizeof(z));                    \
+    return r;                                                                        \
+  }
+
 // ---------------------------------------------------------------------------
 // Numeric helpers
 // ---------------------------------------------------------------------------

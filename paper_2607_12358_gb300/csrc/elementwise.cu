@@ -86,7 +86,7 @@ __global__ void __launch_bounds__(kThreads, 4) drift_partials_kernel(const T* __
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int64_t i = base + u * stride;
-      if (i < nvec) {
+      if (i < nvec && ACID_IN_BOUNDS(kSiteDrift, i * V + V - 1, n)) {
         pr[u] = __ldcs(p4 + i);
         cr[u] = __ldcs(c4 + i);
         if (kApply) rr[u] = __ldcs(r4 + i);
@@ -178,6 +178,7 @@ __global__ void __launch_bounds__(kThreads) add_vec_kernel(const T* __restrict__
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = tid; i < nvec; i += stride) {
+    if (!ACID_IN_BOUNDS(kSiteAdd, i * V + V - 1, n)) continue;
     float x[V], r[V];
     Vec<T>::ld(a + i * V, x);
     Vec<T>::ld(b + i * V, r);
@@ -202,6 +203,7 @@ __global__ void add_mixed8_kernel(const TA* __restrict__ a, const TB* __restrict
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   for (int64_t i = tid; i < n / 8; i += stride) {
+    if (!ACID_IN_BOUNDS(kSiteAdd, 8 * i + 7, n)) continue;
     float x[8];
     load8(a + 8 * i, x);
     if constexpr (READ_B) {
@@ -254,7 +256,7 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     const int c = (i * 32 + lane) * 8;
-    if (c < d) {
+    if (c < d && ACID_IN_BOUNDS(kSiteLayerNorm, row * d + c + 7, rows * d)) {
       const uint4* src = reinterpret_cast<const uint4*>(xr + c);
 #pragma unroll
       for (int k = 0; k < kW; ++k) raw[i][k] = src[k];
@@ -306,7 +308,7 @@ __global__ void __launch_bounds__(kThreads) ln_mod_kernel(const Tin* __restrict_
 #pragma unroll
         for (int j = 0; j < 8; ++j) o[j] = (f[j] - mean) * rstd;
       }
-      store8(yr + c, o);
+      if (ACID_IN_BOUNDS(kSiteLayerNorm, row * d + c + 7, rows * d)) store8(yr + c, o);
     }
   }
 }
@@ -390,7 +392,8 @@ __global__ void __launch_bounds__(32 * kTemniMaxWarps, 1) temni_drift_kernel(con
   const uint64_t prev_policy = l2_policy_evict_first();
   auto issue = [&](int64_t k) {
     const int st = (int)(k % kTemniStages);
-    const int64_t row = rows - 1 - (gw + k * nw);
+    int64_t row = rows - 1 - (gw + k * nw);
+    if (!ACID_IN_BOUNDS(kSiteTemni, row, rows)) row = 0;  // (debug builds) read row 0 instead
     mbar_expect_tx(&wf[st], 2 * row_bytes);
     bulk_load(wr + (size_t)st * 2 * d, xc + row * d, row_bytes, &wf[st]);
     bulk_load_hint(wr + (size_t)st * 2 * d + d, xp + row * d, row_bytes, &wf[st], prev_policy);
@@ -549,6 +552,7 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(const TW* __restrict__ W
   const TW* wr = W + (int64_t)row * k;
   float acc = 0.f;
   for (int c = lane * 8; c < k; c += 256) {
+    if (!ACID_IN_BOUNDS(kSiteGemv, (int64_t)row * k + c + 7, (int64_t)n_out * k)) continue;
     float w[8];
     load8(wr + c, w);
 #pragma unroll
@@ -612,7 +616,7 @@ __global__ void patchify_kernel(const float* __restrict__ lat, TO* __restrict__ 
     const int dt = p % pt; p /= pt;
     const int c = p;
     const int64_t src = (((int64_t)c * F + (f * pt + dt)) * H + (h * ph + dh)) * W + (w * pw + dw);
-    io<TO>::st(tok + i, lat[src]);
+    if (ACID_IN_BOUNDS(kSitePatchify, src, (int64_t)C * F * H * W)) io<TO>::st(tok + i, lat[src]);
   }
 }
 
@@ -638,6 +642,9 @@ __global__ void patchify_split_kernel(const float* __restrict__ lat, __nv_bfloat
     const int dt = p % pt; p /= pt;
     const int c = p;
     const int64_t src = (((int64_t)c * F + (f * pt + dt)) * H + (h * ph + dh)) * W + (w * pw + dw);
+    if (!ACID_IN_BOUNDS(kSitePatchify, src, (int64_t)C * F * H * W) ||
+        !ACID_IN_BOUNDS(kSitePatchify, n * 2 * P + P + p0, total * 2))
+      continue;
     const float x = lat[src];
     const __nv_bfloat16 hi = __float2bfloat16_rn(x);
     tok[n * 2 * P + p0] = hi;
@@ -658,6 +665,7 @@ __global__ void unpatchify_euler_kernel(const float* __restrict__ vtok, float* _
     const int c = (int)(i / ((int64_t)W * H * F));
     const int64_t n = ((int64_t)(f / pt) * Hp + h / ph) * Wp + w / pw;
     const int p = ((c * pt + f % pt) * ph + h % ph) * pw + w % pw;
+    if (!ACID_IN_BOUNDS(kSiteUnpatchify, n * P + p, (int64_t)(F / pt) * Hp * Wp * P)) continue;
     const float v = vtok[n * P + p];
     if (vout) vout[i] = v;
     if (lat) lat[i] = fmaf(dsig, v, lat[i]);
@@ -708,6 +716,8 @@ int grid_for(int64_t work, int per_block = kThreads, int cap = 152 * 16) {
 }
 
 }  // namespace
+
+ACID_BOUNDS_READER(take_bounds_elementwise)
 
 // =========================================================================
 // host launchers

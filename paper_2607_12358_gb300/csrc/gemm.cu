@@ -91,6 +91,11 @@ __device__ __forceinline__ const float2& rope_cs_ptr(const RopeTable& t, const R
   return t.table[off_w + p.w * t.pairs_w + jj];
 }
 __device__ __forceinline__ float2 rope_cs(const RopeTable& t, const RopePos& p, int jj) { return rope_cs_ptr(t, p, jj); }
+// (debug builds) the table entry's index lies inside the table
+__device__ __forceinline__ bool rope_in_bounds(const RopeTable& t, const float2& e) {
+  const int64_t n = (int64_t)t.grid_f * t.pairs_t + (int64_t)t.grid_h * t.pairs_h + (int64_t)t.grid_w * t.pairs_w;
+  return ACID_IN_BOUNDS(kSiteGemmRope, &e - t.table, n);
+}
 
 // Applies the epilogue to the adjacent outputs (grow, col) and (grow, col+1).
 // r0/r1: residual values (read by the caller) for the residual kinds.
@@ -195,7 +200,8 @@ __device__ __forceinline__ void load_chunk_inputs(const GemmDims& g, const EpiDe
 #pragma unroll
     for (int p = 0; p < 8; ++p) {
       const int64_t row = row0 + 4 * p + (lane >> 3);
-      if (row >= g.M) {  // computed but not stored by the epilogue
+      if (row >= g.M || !ACID_IN_BOUNDS(kSiteGemmResidual, row * e.ldr + col + 3, (g.M - 1) * e.ldr + g.N)) {
+        // computed but not stored by the epilogue
 #pragma unroll
         for (int q = 0; q < (R32 ? 4 : 2); ++q) rc.w[p][q] = 0u;
         continue;
@@ -298,7 +304,8 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
       if (col < 2 * e.d && grow >= e.rope_first_video && row0 + 4 * p + (lane >> 3) < g.M) {
         const RopePos pp = rope_pos(e.rope, (int)(grow - e.rope_first_video));
 #pragma unroll
-        for (int q = 0; q < 2; ++q) rcs[p][q] = __ldg(&rope_cs_ptr(e.rope, pp, j0 + q));
+        for (int q = 0; q < 2; ++q)
+          if (rope_in_bounds(e.rope, rope_cs_ptr(e.rope, pp, j0 + q))) rcs[p][q] = __ldg(&rope_cs_ptr(e.rope, pp, j0 + q));
       }
     }
   }
@@ -360,7 +367,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmDims& g, const EpiDev& 
       }
     } else {
       const int64_t row = row0 + rr;
-      if (row >= g.M) continue;
+      if (row >= g.M || !ACID_IN_BOUNDS(kSiteGemmStore, row * g.ldo + col + 3, (g.M - 1) * g.ldo + g.N)) continue;
       if constexpr (O32)
         *reinterpret_cast<float4*>(static_cast<float*>(g.out) + row * g.ldo + col) = make_float4(v[0], v[1], v[2], v[3]);
       else
@@ -428,7 +435,8 @@ __device__ __forceinline__ void epilogue_rows(const GemmDims& g, const EpiDev& e
       const int j0 = (col0 & (e.head_dim - 1)) >> 1;
 #pragma unroll
       for (int k = 0; k < 16; ++k) {
-        const float2 cs = __ldg(&rope_cs_ptr(e.rope, pp, j0 + k));
+        const float2& ce = rope_cs_ptr(e.rope, pp, j0 + k);
+        const float2 cs = rope_in_bounds(e.rope, ce) ? __ldg(&ce) : make_float2(1.f, 0.f);
         float x0, x1;
         f2_unpack(v[k], x0, x1);
         v[k] = f2_pack(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
@@ -1084,6 +1092,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const float* __restrict__
       }
       float a = acc[i][j], b = acc[i][j + 1];
       epi_pair<false>(e, grow, col, a, b, r0, r1);
+      if (!ACID_IN_BOUNDS(kSiteGemmF32, row * ldo + col + 1, (M - 1) * ldo + N)) continue;
       out[row * ldo + col] = a;
       out[row * ldo + col + 1] = b;
     }
@@ -1144,5 +1153,6 @@ acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int
 }
 
 ACID_DEVICE_FLAG_READER(take_device_error_gemm)
+ACID_BOUNDS_READER(take_bounds_gemm)
 
 }  // namespace acid
