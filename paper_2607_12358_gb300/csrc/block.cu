@@ -52,6 +52,8 @@ BlockWs block_ws_layout(const acid_block_desc& d, void* base) {
   if (d.dtype == ACID_BF16 && d.heads > 0) {
     w.attn_part_bytes = attn_part_bytes(d.d / d.heads);
     w.attn_part = b.take<uint8_t>(w.attn_part_bytes);
+    w.splitk_bytes = kSplitKScratchBytes;
+    w.splitk = b.take<uint8_t>(w.splitk_bytes);
   }
   w.kvc = (d.kind == ACID_BLOCK_WAN && d.n_text > 0) ? b.take<uint8_t>(d.n_text * 2 * (int64_t)d.d * es) : nullptr;
   w.bytes = b.off + 1024;
@@ -196,6 +198,8 @@ acid_status block_forward_impl(const acid_block_desc& D, void* x, const float* t
     e.residual = xm + r0 * d;
     e.res_fp32 = true;
     e.out_fp32 = dt == ACID_FP32;
+    e.splitk_ws = ws.splitk;  // FFN2 (K = ffn): a long mainloop
+    e.splitk_bytes = ws.splitk_bytes;
     return e;
   };
 

@@ -34,6 +34,8 @@ struct BlockWs {
   float* xm = nullptr;     // [rows, d] fp32 residual stream between the two branches
   void* attn_part = nullptr;  // attention partial results of a split last wave
   size_t attn_part_bytes = 0;
+  void* splitk = nullptr;     // partial accumulators of a split-K last GEMM round
+  size_t splitk_bytes = 0;
   size_t bytes = 0;
 };
 

@@ -166,6 +166,11 @@ struct GemmDims {
   void* out;
   int64_t ldo;
   int out_fp32;
+  // split-K launches of the pair kernel only: work unit = (tile, split);
+  // split s covers k-blocks [s kb_split, (s + 1) kb_split) and stores its
+  // raw fp32 accumulator at rows s m_pad + row of the partial buffer
+  int splits = 1, kb_split = 0;
+  int64_t m_pad = 0;
 };
 
 // Epilogue of 32-row x 32-column accumulator chunks held by a warp (thread =
@@ -416,8 +421,8 @@ __device__ __forceinline__ void load_bias32(const EpiDev& e, int col0, float* bi
 // makes sure the store that last read this stage has finished reading.
 template <int KIND, bool O32>
 __device__ __forceinline__ void epilogue_rows(const GemmDims& g, const EpiDev& e, const CUtensorMap* tmO,
-                                              uint8_t* stage, int64_t row0, int col0, const uint32_t* r,
-                                              const float* bias) {
+                                              uint8_t* stage, int64_t row0, int64_t store_row0, int col0,
+                                              const uint32_t* r, const float* bias) {
   const int lane = threadIdx.x & 31;
   uint64_t v[16];
 #pragma unroll
@@ -467,7 +472,7 @@ __device__ __forceinline__ void epilogue_rows(const GemmDims& g, const EpiDev& e
   fence_proxy_async_smem();
   __syncwarp();
   if (lane == 0) {
-    tma_store_2d(tmO, stage, col0, (int)row0);
+    tma_store_2d(tmO, stage, col0, (int)store_row0);
     bulk_commit_group();
   }
 }
@@ -477,8 +482,8 @@ __device__ __forceinline__ void epilogue_rows(const GemmDims& g, const EpiDev& e
 // only for the store before last; fp32 output: one 4 KB stage), epilogue_rows.
 template <int KIND, bool O32>
 __device__ __forceinline__ void tma_kind_chunk(const GemmDims& g, const EpiDev& e, const CUtensorMap* tmO,
-                                               uint8_t* stage, uint32_t taddr, int64_t row0, int col0, bool ok,
-                                               int& nstore) {
+                                               uint8_t* stage, uint32_t taddr, int64_t row0, int64_t store_row0,
+                                               int col0, bool ok, int& nstore) {
   const int lane = threadIdx.x & 31;
   uint32_t r[32];
   float bias[32];
@@ -495,7 +500,7 @@ __device__ __forceinline__ void tma_kind_chunk(const GemmDims& g, const EpiDev& 
     if (lane == 0) bulk_wait_group_read<1>();
   }
   __syncwarp();
-  epilogue_rows<KIND, O32>(g, e, tmO, st, row0, col0, r, bias);
+  epilogue_rows<KIND, O32>(g, e, tmO, st, row0, store_row0, col0, r, bias);
   ++nstore;
 }
 
@@ -678,7 +683,7 @@ struct Tc2Cfg {
 };
 static_assert(Tc2Cfg::SMEM <= 232448, "pair GEMM shared memory");
 
-template <int KIND, bool R32, bool O32>
+template <int KIND, bool R32, bool O32, bool SPLIT = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmO, GemmDims g, EpiDev e) {
@@ -698,9 +703,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   const int pair = (int)blockIdx.x >> 1, npairs = (int)gridDim.x >> 1;
-  const int num_kb = (g.K + BK - 1) / BK;
+  const int num_kb = SPLIT ? g.kb_split : (g.K + BK - 1) / BK;
   const int num_n = (g.N + BN - 1) / BN;
   const int num_tiles = (int)((g.M + 2 * BM - 1) / (2 * BM)) * num_n;
+  const int num_units = SPLIT ? num_tiles * g.splits : num_tiles;  // (tile, split) pairs
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
@@ -728,14 +734,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const uint32_t full0 = mapa_shared(smem_u32(full), 0);  // rank 0's full[0]
       int it = 0;
       bool ok = true;
-      for (int tile = pair; ok && tile < num_tiles; tile += npairs) {
+      for (int unit = pair; ok && unit < num_units; unit += npairs) {
+        const int tile = SPLIT ? unit / g.splits : unit;
+        const int kb0 = SPLIT ? (unit % g.splits) * num_kb : 0;
         const int m_tile = tile / num_n, n_tile = tile % num_n;
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES, round = it / C::STAGES;
           if (round > 0 && !mbar_wait(&empty[s], (round - 1) & 1)) { ok = false; break; }
           if (rank == 0) mbar_expect_tx(&full[s], 2 * C::STAGE_BYTES);
-          tma_load_2d_pair(sA + s * C::A_BYTES, &tmA, full0 + 8 * s, kb * BK, m_tile * 2 * BM + (int)rank * BM);
-          tma_load_2d_pair(sB + s * C::B_BYTES, &tmB, full0 + 8 * s, kb * BK, n_tile * BN + (int)rank * (BN / 2));
+          tma_load_2d_pair(sA + s * C::A_BYTES, &tmA, full0 + 8 * s, (kb0 + kb) * BK, m_tile * 2 * BM + (int)rank * BM);
+          tma_load_2d_pair(sB + s * C::B_BYTES, &tmB, full0 + 8 * s, (kb0 + kb) * BK,
+                           n_tile * BN + (int)rank * (BN / 2));
         }
       }
       // After a wait ran out: rank 0 waits (bounded) for the last STAGES
@@ -759,7 +768,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const uint32_t accf_l = smem_u32(acc_full), accf_r = mapa_shared(accf_l, 1);
       int it = 0, local = 0;
       bool ok = true;
-      for (int tile = pair; ok && tile < num_tiles; tile += npairs, ++local) {
+      for (int unit = pair; ok && unit < num_units; unit += npairs, ++local) {
         const int b = local & 1, use = local >> 1;
         if (use > 0 && !mbar_wait_cluster(&acc_empty[b], (use - 1) & 1)) { ok = false; break; }
         tc_fence_after();
@@ -795,7 +804,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     float* stage = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES) + (warp - 2) * C::EPI_STAGE_FLOATS;
     const uint32_t acc_empty0 = mapa_shared(smem_u32(acc_empty), 0);
     int local = 0, nstore = 0;
-    for (int tile = pair; tile < num_tiles; tile += npairs, ++local) {
+    for (int unit = pair; unit < num_units; unit += npairs, ++local) {
+      const int tile = SPLIT ? unit / g.splits : unit;
       const int b = local & 1, use = local >> 1;
       const int m_tile = tile / num_n, n_tile = tile % num_n;
       const bool ok = mbar_wait(&acc_full[b], use & 1);
@@ -804,11 +814,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       if constexpr (kTmaStore<KIND>) {
         constexpr int NC = BN / 64;
         const int cbeg = half * (BN / 2);
+        const int64_t store_row0 = SPLIT ? row0 + (int64_t)(unit % g.splits) * g.m_pad : row0;
 #pragma unroll 1
         for (int i = 0; i < NC; ++i)
           tma_kind_chunk<KIND, O32>(g, e, &tmO, reinterpret_cast<uint8_t*>(stage),
-                                    tmem + lane_base + b * BN + cbeg + 32 * i, row0, n_tile * BN + cbeg + 32 * i, ok,
-                                    nstore);
+                                    tmem + lane_base + b * BN + cbeg + 32 * i, row0, store_row0,
+                                    n_tile * BN + cbeg + 32 * i, ok, nstore);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cluster(acc_empty0 + 8 * b);
@@ -1036,6 +1047,132 @@ acid_status launch_tc2(const void* A, int64_t lda, int64_t M, int K, const void*
   }
 }
 
+// ---------------------------------------------------------------------------
+// Split-K last round of the pair GEMM.  With K long, a persistent launch
+// whose last round keeps only a few CTA pairs busy spends a whole tile's
+// mainloop on it.  The rows that fill whole rounds then run as usual, and
+// the remaining rows run as (tile, k-split) units, one per pair, each storing
+// its raw fp32 accumulator into scratch; splitk_fixup_kernel adds a row's
+// partials in split order and applies the epilogue.
+struct SplitKPlan {
+  int64_t rows_main = 0;  // rows of the ordinary launch (whole 256-row tiles)
+  int splits = 0, kb_split = 0;
+  int64_t m_pad = 0;      // tail rows rounded up to 256 (per-split stride of the scratch)
+};
+
+bool splitk_plan(int64_t M, int N, int K, size_t ws_bytes, int pairs, SplitKPlan* p) {
+  constexpr int64_t bm = 2 * BM;
+  const int64_t n_tiles = (N + Tc2Cfg::BN - 1) / Tc2Cfg::BN, m_tiles = (M + bm - 1) / bm;
+  const int64_t tiles = m_tiles * n_tiles, num_kb = (K + BK - 1) / BK;
+  if (pairs <= 0 || num_kb < 64) return false;  // short mainloops: the last round is cheap
+  const int64_t full = tiles / pairs, last = tiles - full * pairs;
+  if (full < 1 || last == 0 || 2 * last >= pairs) return false;
+  const int64_t rows_main = (full * pairs / n_tiles) * bm;
+  if (rows_main <= 0 || rows_main >= M) return false;
+  const int64_t tail = M - rows_main, tail_tiles = ((tail + bm - 1) / bm) * n_tiles;
+  const int64_t splits = std::min<int64_t>({pairs / tail_tiles, num_kb / 16, 16});
+  if (splits < 3) return false;
+  p->rows_main = rows_main;
+  p->splits = (int)splits;
+  p->kb_split = (int)((num_kb + splits - 1) / splits);
+  p->m_pad = ((tail + bm - 1) / bm) * bm;
+  return (size_t)splits * p->m_pad * N * sizeof(float) <= ws_bytes;
+}
+
+template <int KIND, bool R32, bool O32>
+__global__ void __launch_bounds__(256) splitk_fixup_kernel(const float* __restrict__ part, int splits, int64_t m_pad,
+                                                           int64_t M, int N, void* out, int64_t ldo, EpiDev e) {
+  const int64_t npair = N / 2, total = M * npair;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+    const int64_t row = i / npair;
+    const int col = (int)(i - row * npair) * 2;
+    float a = 0.f, b = 0.f;
+    for (int sp = 0; sp < splits; ++sp) {
+      const float2 v = *reinterpret_cast<const float2*>(part + ((int64_t)sp * m_pad + row) * N + col);
+      a += v.x;
+      b += v.y;
+    }
+    float r0 = 0.f, r1 = 0.f;
+    if constexpr (KIND == EPI_GATED_RES || KIND == EPI_RES) {
+      if constexpr (R32) {
+        const float2 rv = *reinterpret_cast<const float2*>(static_cast<const float*>(e.res) + row * e.ldr + col);
+        r0 = rv.x;
+        r1 = rv.y;
+      } else {
+        const uint32_t rv = *reinterpret_cast<const uint32_t*>(static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + col);
+        r0 = bf16_lo(rv);
+        r1 = bf16_hi(rv);
+      }
+    }
+    epi_pair<true>(e, row + e.row_base, col, a, b, r0, r1);
+    if (!ACID_IN_BOUNDS(kSiteGemmStore, row * ldo + col + 1, (M - 1) * ldo + N)) continue;
+    if constexpr (O32)
+      *reinterpret_cast<float2*>(static_cast<float*>(out) + row * ldo + col) = make_float2(a, b);
+    else
+      *reinterpret_cast<uint32_t*>(static_cast<__nv_bfloat16*>(out) + row * ldo + col) = pack_bf16(a, b);
+  }
+}
+
+template <int KIND, bool R32, bool O32>
+acid_status launch_splitk_fixup(const SplitKPlan& sp, const float* part, int64_t M, int N, void* out, int64_t ldo,
+                                const Epilogue& epi, cudaStream_t s) {
+  const int64_t total = M * (N / 2);
+  const int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)num_sms() * 8);
+  splitk_fixup_kernel<KIND, R32, O32><<<grid, 256, 0, s>>>(part, sp.splits, sp.m_pad, M, N, out, ldo, to_dev(epi));
+  ACID_CHECK_LAUNCH();
+  return ACID_OK;
+}
+
+template <int KIND, bool R32 = false>
+acid_status launch_splitk_fixup_kind(const SplitKPlan& sp, const float* part, int64_t M, int N, void* out,
+                                     int64_t ldo, const Epilogue& epi, cudaStream_t s) {
+  return epi.out_fp32 ? launch_splitk_fixup<KIND, R32, true>(sp, part, M, N, out, ldo, epi, s)
+                      : launch_splitk_fixup<KIND, R32, false>(sp, part, M, N, out, ldo, epi, s);
+}
+
+// The split-K units of the tail rows [M rows of A], then the fixup into out.
+acid_status launch_tc2_splitk(const void* A, int64_t lda, int64_t M, int K, const void* W, int N, void* out,
+                              int64_t ldo, const Epilogue& epi, const SplitKPlan& sp, cudaStream_t s) {
+  using Kern = decltype(&gemm_tc2_kernel<EPI_BIAS, false, true, true>);
+  const Kern kern = gemm_tc2_kernel<EPI_BIAS, false, true, true>;
+  static bool attr_done = false;
+  if (!attr_done) {
+    ACID_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Tc2Cfg::SMEM));
+    attr_done = true;
+  }
+  float* part = static_cast<float*>(epi.splitk_ws);
+  CUtensorMap ta, tb, to;
+  ACID_TRY(make_tmap_bf16(&ta, A, M, K, lda, BM));
+  ACID_TRY(make_tmap_bf16(&tb, W, N, K, K, Tc2Cfg::BN / 2));
+  ACID_TRY(make_tmap_out(&to, part, (int64_t)sp.splits * sp.m_pad, N, N, true));
+  GemmDims g{M, N, K, part, N, 1};
+  g.splits = sp.splits;
+  g.kb_split = sp.kb_split;
+  g.m_pad = sp.m_pad;
+  Epilogue raw;  // the accumulator as it is: no bias, fp32
+  raw.out_fp32 = true;
+  const int64_t units = ((M + 2 * BM - 1) / (2 * BM)) * ((N + Tc2Cfg::BN - 1) / Tc2Cfg::BN) * sp.splits;
+  const int pairs = max_pairs<EPI_BIAS, false, true>();
+  ACID_REQUIRE(pairs > 0, ACID_ERR_CUDA, "linear: no resident CTA pair for the pair GEMM");
+  {
+    ProfScope prof(PROF_LINEAR, 2.0 * (double)M * N * K, s);
+    kern<<<2 * (int)std::min<int64_t>(units, pairs), kGemmThreads, Tc2Cfg::SMEM, s>>>(ta, tb, to, g, to_dev(raw));
+    ACID_CHECK_LAUNCH();
+  }
+  switch (epi.kind) {
+    case EPI_GELU: return launch_splitk_fixup_kind<EPI_GELU>(sp, part, M, N, out, ldo, epi, s);
+    case EPI_ROPE_QKV: return launch_splitk_fixup_kind<EPI_ROPE_QKV>(sp, part, M, N, out, ldo, epi, s);
+    case EPI_GATED_RES:
+      return epi.res_fp32 ? launch_splitk_fixup_kind<EPI_GATED_RES, true>(sp, part, M, N, out, ldo, epi, s)
+                          : launch_splitk_fixup_kind<EPI_GATED_RES, false>(sp, part, M, N, out, ldo, epi, s);
+    case EPI_RES:
+      return epi.res_fp32 ? launch_splitk_fixup_kind<EPI_RES, true>(sp, part, M, N, out, ldo, epi, s)
+                          : launch_splitk_fixup_kind<EPI_RES, false>(sp, part, M, N, out, ldo, epi, s);
+    default: return launch_splitk_fixup_kind<EPI_BIAS>(sp, part, M, N, out, ldo, epi, s);
+  }
+}
+
 // ===========================================================================
 // fp32 SIMT GEMM: 64x64 tile, 16-deep K slices, 4x4 outputs per thread
 // ===========================================================================
@@ -1146,7 +1283,20 @@ acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int
   // M = 32760, pairs are 1-2% faster for N = 4608 / 8960 or K = 8960 and 3%
   // slower for the 1536 x 1536 output projection, whose fp32 residual traffic
   // bounds it as much as its FLOPs do.
-  if (N > 128 && (N > 2048 || K > 2048)) return launch_tc2(A, lda, M, K, W, N, out, ldo, epi, s);
+  if (N > 128 && (N > 2048 || K > 2048)) {
+    SplitKPlan sp;
+    if (epi.splitk_ws != nullptr && aligned(epi.splitk_ws, 128) &&
+        splitk_plan(M, N, K, epi.splitk_bytes, max_pairs<EPI_BIAS, false, true>(), &sp)) {
+      ACID_TRY(launch_tc2(A, lda, sp.rows_main, K, W, N, out, ldo, epi, s));
+      const size_t osz = epi.out_fp32 ? 4 : 2, rsz = epi.res_fp32 ? 4 : 2;
+      Epilogue et = epi;
+      et.row_base += sp.rows_main;
+      if (et.residual) et.residual = static_cast<const uint8_t*>(et.residual) + sp.rows_main * et.ldr * rsz;
+      return launch_tc2_splitk(static_cast<const uint8_t*>(A) + sp.rows_main * lda * 2, lda, M - sp.rows_main, K, W,
+                               N, static_cast<uint8_t*>(out) + sp.rows_main * ldo * osz, ldo, et, sp, s);
+    }
+    return launch_tc2(A, lda, M, K, W, N, out, ldo, epi, s);
+  }
   if (N > 128) return launch_tc<256>(A, lda, M, K, W, N, out, ldo, epi, s);
   if (N > 64) return launch_tc<128>(A, lda, M, K, W, N, out, ldo, epi, s);
   return launch_tc<64>(A, lda, M, K, W, N, out, ldo, epi, s);

@@ -49,7 +49,15 @@ struct Epilogue {
   int64_t rope_first_video = 0;
   int d = 0, head_dim = 0;
   bool out_fp32 = false;           // output dtype fp32 (else the GEMM dtype)
+  // optional device scratch for a split-K last round of the SM-pair GEMM
+  // (long K only); without it the GEMM runs as one launch
+  void* splitk_ws = nullptr;
+  size_t splitk_bytes = 0;
 };
+
+// Scratch that lets a pair GEMM's split-K last round run (a bound for any
+// shape: at most one 256 x 256 fp32 partial tile per resident CTA pair).
+constexpr size_t kSplitKScratchBytes = (size_t)80 * 256 * 256 * 4;
 
 // out[M, N] (row stride ldo) = epilogue(A[M, K] (row stride lda) * W[N, K]^T)
 acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int K, const void* W,
