@@ -37,7 +37,11 @@ def acid():
 
 def _rows(n_total, n_text, seed=0):
     rng = np.random.default_rng(seed)
-    base = {0, 1, 2, 3, n_total - 1, n_total - 2, n_total - 3, n_total - 4, n_total - 60, n_total - 127}
+    # the last rows, and those around 504 and 256 rows from the end: where a
+    # long-K GEMM's split-K last round starts at the Wan shape (32256 of
+    # 32760 rows) and its last 256-row tile
+    base = {0, 1, 2, 3, n_total - 1, n_total - 2, n_total - 3, n_total - 4, n_total - 60, n_total - 127,
+            n_total - 505, n_total - 504, n_total - 503, n_total - 257, n_total - 256}
     if n_text:
         base |= {n_text - 1, n_text, n_text + 1, n_text // 2}
     base |= set(rng.integers(0, n_total, size=24).tolist())
