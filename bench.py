@@ -496,6 +496,22 @@ def run_ours(args) -> None:
     acid_ms = e0.elapsed_time(e1)
     computed = sum(int(x.computed) for x in logs)
 
+    # ---- a step that reuses the cache: time embedding, patch embedding, the
+    # TEMNI drift and the host decision, the cached residual, the final layer
+    # and the Euler update (the method's whole per-step cost when it skips)
+    c5, keep5 = acid.loop_cfg(cfg, n_steps=W + K + 2, forced=[True] + [False] * (W + K + 1))
+    loop5 = acid.Loop(model, c5, text, dev)
+    lat5 = torch.from_numpy(lat0).to(dev)
+    for _ in range(W + 1):
+        loop5.step(lat5, log=False)
+    barrier()
+    e0.record()
+    for _ in range(K):
+        loop5.step(lat5, log=False)
+    e1.record()
+    barrier()
+    skip_ms = max_over_ranks(e0.elapsed_time(e1) / K, world)
+
     # ---- the same every-step-computed generation as one CUDA graph (signal and
     # decision on the device); the wall time includes building and
     # instantiating the graph
@@ -535,6 +551,9 @@ def run_ours(args) -> None:
         "acid_mode": {"steps_per_s": K / (acid_ms / 1000.0), "computed_steps": computed, "of": K,
                       "tau_low": cfg.tau_low, "tau_high": cfg.tau_high, "delta": cfg.delta,
                       "note": "random weights: the skip rate says nothing about a trained model"},
+        "skip_step": {"ms": skip_ms, "frac_of_computed_step": skip_ms / (t_max / K),
+                      "note": "a step whose decision is to reuse: time and patch embedding, TEMNI drift, host "
+                              "decision, cached residual, final layer, Euler update"},
         "graph_mode": {"steps_per_s": job_rate(K, graph_s, world),
                        "note": "the same K steps, every step computed, as one CUDA graph (WHILE over steps, "
                                "IF/ELSE per decision); wall time including graph build and instantiation"},
