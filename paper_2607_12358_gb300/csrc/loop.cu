@@ -476,12 +476,6 @@ struct StepTimer {
   }
 };
 
-// One branch's model evaluation at step st->step: Algorithm 1's decision,
-// then the base method's compute or reuse.  defer_euler = false applies the
-// Euler update to the latent in place; defer_euler = true leaves the latent
-// unchanged and points *v_out at the branch's velocity (fp32, latent layout,
-// inside w).  Fills the step log's fields except ms; does not advance
-// st->step.
 // Patch embedding H_in (fp32) of the latent.  bf16 models: the tokens as
 // bf16 hi + lo parts against the weights repeated along K, one tcgen05 GEMM
 // with fp32 accumulation (the fp32 tokens to within 2^-17 relative); fp32
@@ -500,6 +494,12 @@ static acid_status patch_embed(const acid_model& m, const LoopWs& w, const float
   return linear_forward_f32(w.tokens, sh.P, sh.N, (int)sh.P, m.block.dtype, m.patch.w, sh.d, h_in, sh.d, e, s);
 }
 
+// One branch's model evaluation at step st->step: Algorithm 1's decision,
+// then the base method's compute or reuse.  defer_euler = false applies the
+// Euler update to the latent in place; defer_euler = true leaves the latent
+// unchanged and points *v_out at the branch's velocity (fp32, latent layout,
+// inside w).  Fills the step log's fields except ms; does not advance
+// st->step.
 static acid_status branch_step(const acid_model* m, const acid_loop_cfg* cfg, acid_loop_state* st, float* latent,
                                const LoopWs& w, bool defer_euler, const float** v_out, acid_step_log& lg,
                                cudaStream_t s) {
