@@ -137,7 +137,6 @@ __global__ void __launch_bounds__(kThreads, 4) drift_partials_kernel(const T* __
   }
 }
 
-// Fixed-order reduction of the CTA partials; result = {rel, num, den}.
 // {rel, num, den} of the drift from its two sums (zero denominator: 0 when
 // the numerator is 0, else +inf).
 __device__ __forceinline__ void write_drift_result(double num, double den, double* result) {
@@ -149,6 +148,7 @@ __device__ __forceinline__ void write_drift_result(double num, double den, doubl
   result[2] = den;
 }
 
+// Fixed-order reduction of the CTA partials; result = {rel, num, den}.
 __global__ void __launch_bounds__(kThreads) drift_final_kernel(const double2* __restrict__ partials, int nparts,
                                                                double* __restrict__ result) {
   double n = 0.0, d = 0.0;
