@@ -1,12 +1,15 @@
 // Linear layers of the DiT block.
 //
-// bf16: a tcgen05 GEMM.  One CTA computes a 128 x BN output tile with the
-// fp32 accumulator in tensor memory (TMEM).  Warp 0 streams 128x64 A and
-// BNx64 B tiles with TMA (128-byte swizzle) through a STAGES-deep mbarrier
-// ring; warp 1 issues tcgen05.mma (M=128, N=BN, K=16) from one thread;
-// warps 2-5 wait for the accumulator, read it back with tcgen05.ld (one
-// thread per output row) and apply the fused epilogue (bias, GELU-tanh,
-// 3D RoPE of q/k, gated or plain residual) before storing.
+// bf16: persistent tcgen05 GEMMs.  A CTA (or, for N or K above 2048, a pair
+// of CTAs on two SMs with tcgen05.mma.cta_group::2) computes 128 x BN (pair:
+// 256 x 256) output tiles with the fp32 accumulator in tensor memory (TMEM),
+// double-buffered.  Warp 0 streams the A and B tiles with TMA (128-byte
+// swizzle) through a STAGES-deep mbarrier ring; warp 1 issues tcgen05.mma
+// from one thread; warps 2-9 read the accumulator back with tcgen05.ld (one
+// thread per output row) and apply the fused epilogue (bias, GELU-tanh, 3D
+// RoPE of q/k, gated or plain residual) before storing.  Long-K pair GEMMs
+// inside a block can finish their last round as split-K units (see
+// splitk_plan).
 //
 // fp32: a register-tiled SIMT GEMM with the same epilogue (the fp32 mode's
 // 1e-4 tolerance rules out tf32 tensor cores).
