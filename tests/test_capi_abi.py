@@ -46,6 +46,18 @@ def test_every_declared_function_is_exported(lib):
         assert hasattr(lib, n)
 
 
+def test_debug_build_exports_the_same_boundary():
+    """The debug build (kernel memory-index checks compiled in) builds from
+    the same sources without a GPU and exports every declared function."""
+    from paper_2607_12358_gb300 import build as b
+
+    so = b.build(debug=True)
+    out = subprocess.run(["nm", "-D", "--defined-only", so], capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\sT\s(acid_[a-z0-9_]+)$", out, flags=re.M))
+    missing = [n for n in _declared_functions() if n not in exported]
+    assert not missing, missing
+
+
 def test_version_and_clean_error(lib):
     assert b"sm_103a" in lib.acid_version()
     assert lib.acid_last_error() == b""
