@@ -1283,10 +1283,15 @@ acid_status linear_forward(int dtype, const void* A, int64_t lda, int64_t M, int
   // the zero-filled columns of a partial last tile (N = 1920: 7% extra MMA
   // work, against about 1.6x the throughput).
   // SM pairs where the tiles' mainloop is long enough to matter: measured at
-  // M = 32760, pairs are 1-2% faster for N = 4608 / 8960 or K = 8960 and 3%
-  // slower for the 1536 x 1536 output projection, whose fp32 residual traffic
-  // bounds it as much as its FLOPs do.
-  if (N > 128 && (N > 2048 || K > 2048)) {
+  // M = 32760, pairs are 1-2% faster for N = 4608 / 8960 or K = 8960 and 2-3%
+  // slower for the 1536 x 1536 gated-residual output projection, whose
+  // residual traffic bounds it as much as its FLOPs do.
+  // Kinds without a residual leave through the pair kernel's accumulator-
+  // layout epilogue, which makes pairs faster from N = 1024 on (measured at
+  // M = 32760: cross-attention query 1535 -> 1565 TFLOP/s, the K = 128 patch
+  // embedding 40 -> 32 us); the residual kinds stay on single SMs up to 2048.
+  const bool no_res = epi.kind == EPI_BIAS || epi.kind == EPI_GELU || epi.kind == EPI_ROPE_QKV;
+  if (N > 128 && (N > 2048 || K > 2048 || (no_res && N >= 1024))) {
     SplitKPlan sp;
     if (epi.splitk_ws != nullptr && aligned(epi.splitk_ws, 128) &&
         splitk_plan(M, N, K, epi.splitk_bytes, max_pairs<EPI_BIAS, false, true>(), &sp)) {
